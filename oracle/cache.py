@@ -1,0 +1,91 @@
+"""Reference thin-key / full-value KV cache writes and the int8 key quantiser.
+
+TEST INFRASTRUCTURE ONLY (see oracle/attention.py): used by tests, smoke()
+and the CPU legs of bench.py, never by the product path.
+
+Cache content (paper, Section 2.4, Eqs. 8-9, and the remark after the
+absorbed-query equation in Section 2.3): per token and kv head the cache
+holds an r-wide thin key and a d_v-wide value.  Appending T new tokens to
+sequence b writes logical positions seq_lens[b] .. seq_lens[b]+T-1.
+
+Contiguous layout: k[B][H_kv][cap][r], v[B][H_kv][cap][d_v].
+Paged layout: pools k[P][H_kv][page_size][r], v[P][H_kv][page_size][d_v];
+logical position t of sequence b lives in page page_table[b][t // page_size]
+at slot t % page_size.
+
+int8 keys (the paper's composition with key quantisation, Section 6,
+"Flash Attention and composability"; the paper fixes no scheme).  Reading:
+symmetric per-token, per-kv-head absmax quantisation in fp32,
+    amax  = max_c |k_c|
+    scale = amax / 127            (one IEEE binary32 division, round to nearest)
+    code  = clamp(rint(k_c / scale), -127, 127)   (binary32 division, ties to even)
+and amax == 0 gives scale 0 and all-zero codes.  Dequantised key: code * scale.
+"""
+
+from __future__ import annotations
+
+import numpy as np
+
+
+def quantize_int8_per_token(k) -> tuple[np.ndarray, np.ndarray]:
+    """Quantise keys [..., r] (float32 values) to int8 codes [..., r] and fp32 scales [...].
+
+    All arithmetic is binary32 (numpy float32 division is IEEE round-to-nearest;
+    np.rint rounds half to even).
+    """
+    k32 = np.asarray(k, dtype=np.float32)
+    amax = np.max(np.abs(k32), axis=-1)
+    scale = (amax / np.float32(127.0)).astype(np.float32)
+    safe = np.where(scale == 0, np.float32(1.0), scale).astype(np.float32)
+    ratio = (k32 / safe[..., None]).astype(np.float32)
+    codes = np.clip(np.rint(ratio), -127, 127).astype(np.int8)
+    codes[scale == 0] = 0
+    return codes, scale
+
+
+def append_contiguous(k_cache, v_cache, seq_lens, k_new, v_new, k_scale=None):
+    """Write new tokens into contiguous caches (in place) and return them.
+
+    k_cache: [B, H_kv, cap, r] (values, or int8 codes when k_scale [B, H_kv, cap]
+    is given); v_cache: [B, H_kv, cap, d_v]; k_new: [B, H_kv, T, r] float32
+    values; v_new: [B, H_kv, T, d_v].  Positions beyond cap are an error.
+    """
+    B, _, T, _ = np.asarray(k_new).shape
+    cap = k_cache.shape[2]
+    for b in range(B):
+        p0 = int(seq_lens[b])
+        if p0 + T > cap:
+            raise ValueError(f"sequence {b}: {p0}+{T} tokens exceed capacity {cap}")
+        if k_scale is None:
+            k_cache[b, :, p0:p0 + T] = k_new[b]
+        else:
+            codes, sc = quantize_int8_per_token(k_new[b])
+            k_cache[b, :, p0:p0 + T] = codes
+            k_scale[b, :, p0:p0 + T] = sc
+        v_cache[b, :, p0:p0 + T] = v_new[b]
+    return k_cache, v_cache, k_scale
+
+
+def append_paged(k_pool, v_pool, page_table, seq_lens, page_size, k_new, v_new,
+                 k_scale_pool=None):
+    """Write new tokens into paged pools (in place) and return them.
+
+    Pools: [P, H_kv, page_size, r|d_v]; scales [P, H_kv, page_size];
+    page_table: [B, max_pages].
+    """
+    B, _, T, _ = np.asarray(k_new).shape
+    for b in range(B):
+        p0 = int(seq_lens[b])
+        if k_scale_pool is not None:
+            codes, sc = quantize_int8_per_token(k_new[b])
+        for t in range(T):
+            pos = p0 + t
+            page = int(page_table[b][pos // page_size])
+            slot = pos % page_size
+            if k_scale_pool is None:
+                k_pool[page, :, slot] = k_new[b][:, t]
+            else:
+                k_pool[page, :, slot] = codes[:, t]
+                k_scale_pool[page, :, slot] = sc[:, t]
+            v_pool[page, :, slot] = v_new[b][:, t]
+    return k_pool, v_pool, k_scale_pool
