@@ -1,0 +1,191 @@
+/*
+ * tk.h -- C ABI of the thin-key ("factored-key") attention library for
+ * GB300 (sm_103a).
+ *
+ * The method (arxiv 2603.04427, "Thin Keys, Full Values"):
+ *   Section 2.1, Eqs. 1-4: per head, out = softmax(Q K^T * scale) V where
+ *   queries and keys are r wide (the selection dimension d_select/h) and
+ *   values keep the full head width d_v.  The paper's scale is
+ *   1/sqrt(r) (Eq. 4); it is an explicit argument here.
+ *   Section 2.3 (thin-key and absorbed-query equations): only the r-wide
+ *   keys are cached; queries arrive already projected to r.
+ *   Section 2.4, Eqs. 8-9: the cache holds r + d_v values per token and
+ *   kv head.
+ *   Section 3.4 / 3.5: thin keys compose with GQA; query head h reads kv
+ *   head h / (h_q / h_kv).
+ *   Section 6 ("Flash Attention and composability"): thin keys compose
+ *   with key quantisation; here int8 keys with one fp32 absmax scale per
+ *   token and kv head.
+ *
+ * Conventions for every entry point:
+ *   - Device pointers are raw CUDA device addresses on the current device.
+ *     The caller owns every buffer; the library allocates no device memory.
+ *   - All work is enqueued on `stream` (a cudaStream_t; NULL = the legacy
+ *     default stream) and is asynchronous: no call synchronises, except
+ *     tk_get_device_error.
+ *   - Argument errors are detected on the host and returned before anything
+ *     is launched.  Launch failures return TK_ERR_CUDA.  Bad values that
+ *     only the device sees (a page id out of range, a seq_len beyond the
+ *     capacity) are clamped to a safe value, recorded in a device error
+ *     word and reported by tk_get_device_error; the output is then
+ *     unspecified but no access leaves the caller's buffers.
+ *   - tk_last_error() returns a human-readable reason for the last non-OK
+ *     status returned on the calling host thread.
+ *   - Tensors are dense, row-major, innermost dimension last, with base
+ *     addresses aligned to 16 bytes.
+ *
+ * Cache layouts (owned by the caller, described by tk_cache_desc):
+ *   contiguous (page_size == 0):
+ *     k_cache  [batch][h_kv][capacity][r]   bf16, or int8 codes
+ *     k_scale  [batch][h_kv][capacity]      fp32 (int8 keys only)
+ *     v_cache  [batch][h_kv][capacity][d_v] bf16
+ *   paged (page_size > 0): pools shared by all sequences
+ *     k_cache  [num_pages][h_kv][page_size][r]
+ *     k_scale  [num_pages][h_kv][page_size]
+ *     v_cache  [num_pages][h_kv][page_size][d_v]
+ *     page_table [batch][max_pages_per_seq] int32: logical token t of
+ *     sequence b lives in page page_table[b][t / page_size], slot
+ *     t % page_size.
+ */
+#ifndef TK_H_
+#define TK_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define TK_ABI_VERSION 1
+
+typedef enum tk_status {
+  TK_OK = 0,
+  TK_ERR_INVALID_ARG = 1, /* null/misaligned pointer, inconsistent sizes        */
+  TK_ERR_UNSUPPORTED = 2, /* valid request this build has no kernel for         */
+  TK_ERR_WORKSPACE = 3,   /* workspace missing, misaligned or too small         */
+  TK_ERR_CUDA = 4,        /* a CUDA runtime / driver call failed                */
+  TK_ERR_DEVICE = 5       /* a kernel recorded a bad index or a timed-out wait  */
+} tk_status;
+
+typedef enum tk_dtype {
+  TK_BF16 = 0, /* bfloat16                                  */
+  TK_F32 = 1,  /* IEEE binary32                             */
+  TK_I8 = 2    /* int8 key codes (value = code * k_scale)   */
+} tk_dtype;
+
+/* Shape of a thin-key / full-value cache.
+ *   batch, h_q, h_kv : sequences, query heads, kv heads (h_q % h_kv == 0,
+ *                      h_q / h_kv in {1, 2, 4, 8})
+ *   r                : thin key width per head, in {16, 32, 64, 128}
+ *   d_v              : value width per head, in {64, 128}
+ *   capacity         : contiguous only: token slots per (sequence, kv head),
+ *                      a positive multiple of 16
+ *   page_size        : 0 for contiguous, else tokens per page in
+ *                      {16, 32, 64, 128, 256}
+ *   num_pages        : paged only: pages in each pool
+ *   max_pages_per_seq: paged only: columns of the page table
+ *   k_dtype          : TK_BF16 or TK_I8                                      */
+typedef struct tk_cache_desc {
+  int32_t batch;
+  int32_t h_q;
+  int32_t h_kv;
+  int32_t r;
+  int32_t d_v;
+  int32_t capacity;
+  int32_t page_size;
+  int32_t num_pages;
+  int32_t max_pages_per_seq;
+  int32_t k_dtype;
+} tk_cache_desc;
+
+/* Append n_new tokens to every sequence of the cache (Section 2.3: the
+ * thin keys k' = x W_K' are what the cache stores; Section 2.4: each token
+ * adds r + d_v values per kv head).
+ *   k_new    : device bf16 [batch][h_kv][n_new][r]    new thin keys
+ *   v_new    : device bf16 [batch][h_kv][n_new][d_v]  new values
+ *   seq_lens : device int32 [batch], tokens already cached per sequence;
+ *              token t of the new block goes to position seq_lens[b] + t.
+ *              Not modified: the caller advances it (e.g. += n_new on the
+ *              same stream) before the next call.
+ *   k_scale  : device fp32 per-token scales (int8 keys only, else NULL).
+ *   page_table: device int32 [batch][max_pages_per_seq] (paged only, else NULL).
+ * int8 keys are quantised per (token, kv head): amax = max|k|,
+ * scale = amax / 127 (binary32 division, round to nearest), code =
+ * clamp(rint(k / scale), -127, 127) (binary32 division, ties to even);
+ * amax == 0 stores scale 0 and zero codes.
+ * n_new == 0 is a no-op.  Positions beyond the capacity (contiguous) or
+ * beyond max_pages_per_seq * page_size (paged) are not written and set the
+ * device error word.                                                        */
+tk_status tk_kv_append(const tk_cache_desc* desc, void* k_cache, void* v_cache, float* k_scale,
+                       const int32_t* page_table, const int32_t* seq_lens, const void* k_new,
+                       const void* v_new, int32_t n_new, void* stream);
+
+/* Causal (or full) prefill attention over one prompt per sequence
+ * (Section 2.1, Eqs. 1-4; prefill is the compute-bound case of Appendix E).
+ *   q   : device bf16 [batch][h_q][seq][r]
+ *   k   : device bf16 [batch][h_kv][seq][r]
+ *   v   : device bf16 [batch][h_kv][seq][d_v]
+ *   out : device [batch][h_q][seq][d_v], bf16 (out_dtype TK_BF16, round to
+ *         nearest even) or fp32 (TK_F32)
+ *   scale: multiplies q.k (the paper uses 1/sqrt(r))
+ *   causal: nonzero = query i attends to keys 0..i (top-left aligned);
+ *           zero = every query attends to all seq keys.
+ * Shapes: r in {16, 32, 64, 128}, d_v in {64, 128}, h_q % h_kv == 0,
+ * seq >= 0 (seq == 0 is a no-op).  Scores and the weighted sum accumulate
+ * in fp32 on the tensor cores; the softmax weights enter the second
+ * product rounded to bf16.                                                  */
+tk_status tk_attn_prefill(const void* q, const void* k, const void* v, void* out,
+                          int32_t out_dtype, int32_t batch, int32_t h_q, int32_t h_kv,
+                          int32_t seq, int32_t r, int32_t d_v, float scale, int32_t causal,
+                          void* stream);
+
+/* Bytes of decode workspace needed for a cache of this shape when no
+ * sequence is longer than max_seq_len, on the current device (the split of
+ * the context depends on its SM count).  0 means the arguments are invalid.
+ * The workspace must be zero-filled once before its first use; every
+ * completed tk_attn_decode call leaves it zero-filled again, so it can be
+ * reused by later calls in stream order (never by two calls that may run
+ * concurrently).                                                            */
+size_t tk_decode_workspace_size(const tk_cache_desc* desc, int32_t max_seq_len);
+
+/* Single-token decode attention over the cache (Section 2.1, Eq. 4 with one
+ * query row; the bandwidth-bound case of Section 4.2).
+ *   q        : device bf16 [batch][h_q][r], one query token per sequence
+ *   seq_lens : device int32 [batch], context length of each sequence
+ *              (0 gives a zero output row)
+ *   max_seq_len: host upper bound of seq_lens, sizes the launch; a larger
+ *              device value is clamped to it and flagged.
+ *   out      : device [batch][h_q][d_v], TK_F32 or TK_BF16
+ *   scale    : multiplies q.k (for int8 keys, q.(code * k_scale))
+ *   workspace: device scratch of tk_decode_workspace_size bytes, aligned to
+ *              256 bytes (see tk_decode_workspace_size).
+ * The context is split into fixed token ranges processed in parallel and
+ * merged in the same launch; results are deterministic run to run.        */
+tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k_cache,
+                         const void* v_cache, const float* k_scale, const int32_t* page_table,
+                         const int32_t* seq_lens, int32_t max_seq_len, void* out,
+                         int32_t out_dtype, float scale, void* workspace,
+                         size_t workspace_bytes, void* stream);
+
+/* Synchronise `stream`, then read and clear the device error word of the
+ * current device: *code_out = 0 if no kernel recorded an error since the
+ * last call, else a nonzero code (1 = index out of range, 2 = a wait timed
+ * out).  Returns TK_ERR_DEVICE when the word was nonzero.                  */
+tk_status tk_get_device_error(int32_t* code_out, void* stream);
+
+/* Static string naming a status code.                                      */
+const char* tk_status_string(tk_status status);
+
+/* Reason for the last non-OK status returned on this host thread ("" if
+ * none).  The pointer stays valid until the next call on this thread.      */
+const char* tk_last_error(void);
+
+/* TK_ABI_VERSION of the loaded library.                                     */
+int32_t tk_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TK_H_ */

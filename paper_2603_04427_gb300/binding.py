@@ -1,0 +1,235 @@
+"""ctypes binding of ``libtk.so`` (include/tk.h), one Python function per entry point.
+
+Argument marshalling only: each function checks that the torch tensors it
+is given have the dtype, device and contiguity the C ABI expects, passes
+their ``data_ptr()`` and the current CUDA stream, and raises ``TkError`` on
+a non-OK status.  Every step of the computation runs in the library's
+kernels; there is no CPU or PyTorch fallback, and a missing library raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+from dataclasses import dataclass
+
+import torch
+
+TK_OK, TK_ERR_INVALID_ARG, TK_ERR_UNSUPPORTED, TK_ERR_WORKSPACE, TK_ERR_CUDA, TK_ERR_DEVICE = range(6)
+TK_BF16, TK_F32, TK_I8 = 0, 1, 2
+
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtk.so")
+
+EXPORTED = ("tk_kv_append", "tk_attn_prefill", "tk_decode_workspace_size", "tk_attn_decode",
+            "tk_get_device_error", "tk_status_string", "tk_last_error", "tk_abi_version")
+
+
+class TkError(RuntimeError):
+    def __init__(self, status: int, where: str, detail: str):
+        super().__init__(f"{where}: {_status_name(status)}: {detail}")
+        self.status = status
+
+
+class tk_cache_desc(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "batch", "h_q", "h_kv", "r", "d_v", "capacity", "page_size", "num_pages",
+        "max_pages_per_seq", "k_dtype")]
+
+
+_lib = None
+
+
+def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Load libtk.so once and declare the C signatures; raises if it is missing."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is not built; run `python -m paper_2603_04427_gb300.build` "
+                           "(or __graft_entry__.build()) first")
+    L = ctypes.CDLL(path)
+    vp, i32, f32, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_float, ctypes.c_size_t
+    dp = ctypes.POINTER(tk_cache_desc)
+    sig = {
+        "tk_kv_append": (i32, [dp, vp, vp, vp, vp, vp, vp, vp, i32, vp]),
+        "tk_attn_prefill": (i32, [vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, i32, vp]),
+        "tk_decode_workspace_size": (sz, [dp, i32]),
+        "tk_attn_decode": (i32, [dp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp, sz, vp]),
+        "tk_get_device_error": (i32, [ctypes.POINTER(i32), vp]),
+        "tk_status_string": (ctypes.c_char_p, [i32]),
+        "tk_last_error": (ctypes.c_char_p, []),
+        "tk_abi_version": (i32, []),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(L, name)
+        fn.restype, fn.argtypes = res, args
+    _lib = L
+    return L
+
+
+def _status_name(s: int) -> str:
+    names = {0: "TK_OK", 1: "TK_ERR_INVALID_ARG", 2: "TK_ERR_UNSUPPORTED", 3: "TK_ERR_WORKSPACE",
+             4: "TK_ERR_CUDA", 5: "TK_ERR_DEVICE"}
+    return names.get(s, f"status {s}")
+
+
+def _check(status: int, where: str):
+    if status != TK_OK:
+        raise TkError(status, where, load_library().tk_last_error().decode())
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need(t, dtype, name, device=None):
+    if t is None:
+        return
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if device is not None and t.device != device:
+        raise ValueError(f"{name} is on {t.device}, expected {device}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+# ------------------------------------------------------------------ cache helper
+
+@dataclass
+class ThinKeyCache:
+    """Caller-owned thin-key / full-value cache tensors plus their descriptor.
+
+    Contiguous: k [B, H_kv, cap, r] (bf16 or int8), k_scale [B, H_kv, cap] fp32,
+    v [B, H_kv, cap, d_v] bf16.  Paged: pools [P, H_kv, page_size, ...] and a
+    page table [B, max_pages] int32.
+    """
+    desc: tk_cache_desc
+    k: torch.Tensor
+    v: torch.Tensor
+    k_scale: torch.Tensor | None = None
+    page_table: torch.Tensor | None = None
+
+    @staticmethod
+    def allocate(batch, h_q, h_kv, r, d_v, capacity=0, page_size=0, num_pages=0,
+                 page_table=None, k_int8=False, device="cuda", fill=0):
+        if page_size:
+            if page_table is None:
+                raise ValueError("a paged cache needs a page table")
+            page_table = page_table.to(device=device, dtype=torch.int32).contiguous()
+            lead = (num_pages, h_kv, page_size)
+            max_pages = page_table.shape[1]
+        else:
+            lead = (batch, h_kv, capacity)
+            max_pages = 0
+        kd = torch.int8 if k_int8 else torch.bfloat16
+        k = torch.full(lead + (r,), fill, dtype=kd, device=device)
+        v = torch.full(lead + (d_v,), fill, dtype=torch.bfloat16, device=device)
+        ks = torch.zeros(lead, dtype=torch.float32, device=device) if k_int8 else None
+        desc = tk_cache_desc(batch, h_q, h_kv, r, d_v, 0 if page_size else capacity, page_size,
+                             num_pages if page_size else 0, max_pages,
+                             TK_I8 if k_int8 else TK_BF16)
+        return ThinKeyCache(desc, k, v, ks, page_table)
+
+
+# ------------------------------------------------------------------ entry points
+
+def tk_abi_version() -> int:
+    return int(load_library().tk_abi_version())
+
+
+def tk_status_string(status: int) -> str:
+    return load_library().tk_status_string(status).decode()
+
+
+def tk_last_error() -> str:
+    return load_library().tk_last_error().decode()
+
+
+def tk_kv_append(cache: ThinKeyCache, k_new, v_new, seq_lens, stream=None):
+    """Append k_new [B, H_kv, T, r] / v_new [B, H_kv, T, d_v] (bf16) at seq_lens[b]."""
+    d = cache.desc
+    dev = cache.k.device
+    _need(k_new, torch.bfloat16, "k_new", dev)
+    _need(v_new, torch.bfloat16, "v_new", dev)
+    _need(seq_lens, torch.int32, "seq_lens", dev)
+    T = k_new.shape[2]
+    if tuple(k_new.shape) != (d.batch, d.h_kv, T, d.r) or tuple(v_new.shape) != (d.batch, d.h_kv, T, d.d_v):
+        raise ValueError(f"k_new {tuple(k_new.shape)} / v_new {tuple(v_new.shape)} do not match the cache")
+    L = load_library()
+    _check(L.tk_kv_append(ctypes.byref(d), _ptr(cache.k), _ptr(cache.v), _ptr(cache.k_scale),
+                          _ptr(cache.page_table), _ptr(seq_lens), _ptr(k_new), _ptr(v_new), T,
+                          _stream(stream)), "tk_kv_append")
+
+
+def tk_decode_workspace_size(desc: tk_cache_desc, max_seq_len: int) -> int:
+    n = int(load_library().tk_decode_workspace_size(ctypes.byref(desc), int(max_seq_len)))
+    if n == 0:
+        raise TkError(TK_ERR_INVALID_ARG, "tk_decode_workspace_size", tk_last_error())
+    return n
+
+
+def decode_workspace(desc: tk_cache_desc, max_seq_len: int, device="cuda") -> torch.Tensor:
+    """A zero-filled workspace of the size tk_attn_decode needs (torch owns the memory)."""
+    return torch.zeros(tk_decode_workspace_size(desc, max_seq_len), dtype=torch.uint8, device=device)
+
+
+def tk_attn_decode(cache: ThinKeyCache, q, seq_lens, max_seq_len: int, out, workspace,
+                   scale: float | None = None, stream=None):
+    """One decode step: q [B, H_q, r] bf16 -> out [B, H_q, d_v] (fp32 or bf16)."""
+    d = cache.desc
+    dev = cache.k.device
+    _need(q, torch.bfloat16, "q", dev)
+    _need(seq_lens, torch.int32, "seq_lens", dev)
+    _need(workspace, torch.uint8, "workspace", dev)
+    if out.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("out must be float32 or bfloat16")
+    _need(out, out.dtype, "out", dev)
+    if tuple(q.shape) != (d.batch, d.h_q, d.r) or tuple(out.shape) != (d.batch, d.h_q, d.d_v):
+        raise ValueError(f"q {tuple(q.shape)} / out {tuple(out.shape)} do not match the cache")
+    scale = 1.0 / math.sqrt(d.r) if scale is None else float(scale)
+    L = load_library()
+    _check(L.tk_attn_decode(ctypes.byref(d), _ptr(q), _ptr(cache.k), _ptr(cache.v),
+                            _ptr(cache.k_scale), _ptr(cache.page_table), _ptr(seq_lens),
+                            int(max_seq_len), _ptr(out),
+                            TK_F32 if out.dtype == torch.float32 else TK_BF16, scale,
+                            _ptr(workspace), workspace.numel(), _stream(stream)), "tk_attn_decode")
+    return out
+
+
+def tk_attn_prefill(q, k, v, out, scale: float | None = None, causal: bool = True, stream=None):
+    """Prefill: q [B, H_q, S, r], k [B, H_kv, S, r], v [B, H_kv, S, d_v] bf16 -> out [B, H_q, S, d_v]."""
+    dev = q.device
+    for t, n in ((q, "q"), (k, "k"), (v, "v")):
+        _need(t, torch.bfloat16, n, dev)
+    if out.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("out must be float32 or bfloat16")
+    _need(out, out.dtype, "out", dev)
+    B, hq, S, r = q.shape
+    hkv, dv = k.shape[1], v.shape[3]
+    if tuple(k.shape) != (B, hkv, S, r) or tuple(v.shape) != (B, hkv, S, dv) or \
+            tuple(out.shape) != (B, hq, S, dv):
+        raise ValueError("q / k / v / out shapes are inconsistent")
+    scale = 1.0 / math.sqrt(r) if scale is None else float(scale)
+    L = load_library()
+    _check(L.tk_attn_prefill(_ptr(q), _ptr(k), _ptr(v), _ptr(out),
+                             TK_F32 if out.dtype == torch.float32 else TK_BF16,
+                             B, hq, hkv, S, r, dv, scale, 1 if causal else 0, _stream(stream)),
+           "tk_attn_prefill")
+    return out
+
+
+def tk_get_device_error(stream=None) -> int:
+    """Synchronise the stream and return (and clear) the device error word (0 = none)."""
+    code = ctypes.c_int32(0)
+    st = load_library().tk_get_device_error(ctypes.byref(code), _stream(stream))
+    if st not in (TK_OK, TK_ERR_DEVICE):
+        _check(st, "tk_get_device_error")
+    return int(code.value)

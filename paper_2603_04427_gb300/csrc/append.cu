@@ -1,0 +1,136 @@
+// KV-cache append: writes n_new thin-key rows (r wide) and value rows (d_v
+// wide) per (sequence, kv head) at logical positions seq_lens[b] + t.
+//
+// Paper: Section 2.3 (the thin keys k' = x W_K' are what the cache keeps) and
+// Section 2.4, Eqs. 8-9 (r + d_v values per token and kv head).  The int8
+// variant is the composition with key quantisation of Section 6; the scheme
+// (symmetric absmax per token and kv head, fp32 scale) is this library's
+// reading: scale = amax / 127, code = clamp(rint(k / scale), -127, 127), both
+// divisions in IEEE binary32 (this file is compiled without fast-math).
+//
+// One warp per (b, g, t): 16-byte vector loads and stores for bf16 rows; for
+// int8 keys a warp max-reduction gives amax.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace tk {
+namespace {
+
+constexpr int kWarps = 4;
+
+template <int R, int DV, bool KI8>
+__global__ void __launch_bounds__(kWarps * 32) append_kernel(const AppendParams p) {
+  const int lane = threadIdx.x & 31;
+  const long wg = static_cast<long>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
+  const long total = static_cast<long>(p.B) * p.Hkv * p.T;
+  if (wg >= total) return;
+  const int t = static_cast<int>(wg % p.T);
+  const int g = static_cast<int>((wg / p.T) % p.Hkv);
+  const int b = static_cast<int>(wg / (static_cast<long>(p.T) * p.Hkv));
+  const int pos = p.seq_lens[b] + t;
+
+  size_t row;  // destination row in the cache / pool
+  if (p.page_size == 0) {
+    if (pos < 0 || pos >= p.capacity) {
+      if (lane == 0) record_error(p.err, TK_DEVERR_INDEX);
+      return;
+    }
+    row = (static_cast<size_t>(b) * p.Hkv + g) * p.capacity + pos;
+  } else {
+    const int pidx = pos >> p.page_shift;
+    if (pos < 0 || pidx >= p.max_pages) {
+      if (lane == 0) record_error(p.err, TK_DEVERR_INDEX);
+      return;
+    }
+    const int page = p.page_table[static_cast<size_t>(b) * p.max_pages + pidx];
+    if (page < 0 || page >= p.num_pages) {
+      if (lane == 0) record_error(p.err, TK_DEVERR_INDEX);
+      return;
+    }
+    row = (static_cast<size_t>(page) * p.Hkv + g) * p.page_size + (pos & (p.page_size - 1));
+  }
+  const size_t src = (static_cast<size_t>(b) * p.Hkv + g) * p.T + t;
+
+  // Values: d_v bf16 = 2 * DV bytes, 16 bytes per lane.
+  {
+    constexpr int NV = 2 * DV / 16;
+    const uint4* s = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(p.v_new) +
+                                                    src * 2 * DV);
+    uint4* d = reinterpret_cast<uint4*>(static_cast<unsigned char*>(p.v) + row * 2 * DV);
+    if (lane < NV) d[lane] = s[lane];
+  }
+  if constexpr (!KI8) {
+    constexpr int NK = 2 * R / 16;
+    const uint4* s = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(p.k_new) +
+                                                    src * 2 * R);
+    uint4* d = reinterpret_cast<uint4*>(static_cast<unsigned char*>(p.k) + row * 2 * R);
+    if (lane < NK) d[lane] = s[lane];
+  } else {
+    // Each lane holds EPL = ceil(R / 32) consecutive key elements.
+    constexpr int EPL = R >= 32 ? R / 32 : 1;
+    const __nv_bfloat16* s = static_cast<const __nv_bfloat16*>(p.k_new) + src * R;
+    float x[EPL];
+    float amax = 0.f;
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) {
+      const int c = lane * EPL + e;
+      x[e] = c < R ? __bfloat162float(s[c]) : 0.f;
+      amax = fmaxf(amax, fabsf(x[e]));
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+    const float scale = amax / 127.0f;  // IEEE binary32 division
+    int8_t* d = static_cast<int8_t*>(p.k) + row * R;
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) {
+      const int c = lane * EPL + e;
+      if (c < R) {
+        float code = 0.f;
+        if (scale != 0.f) code = fminf(fmaxf(rintf(x[e] / scale), -127.f), 127.f);
+        d[c] = static_cast<int8_t>(code);
+      }
+    }
+    if (lane == 0) p.k_scale[row] = scale;
+  }
+}
+
+template <int R, int DV, bool KI8>
+cudaError_t launch_t(const AppendParams& p, cudaStream_t s) {
+  const long warps = static_cast<long>(p.B) * p.Hkv * p.T;
+  const long blocks = (warps + kWarps - 1) / kWarps;
+  if (blocks > 0x7fffffffL) return cudaErrorInvalidConfiguration;
+  append_kernel<R, DV, KI8><<<static_cast<unsigned>(blocks), kWarps * 32, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+template <int R, bool KI8>
+cudaError_t by_dv(const AppendParams& p, cudaStream_t s, int* uns) {
+  switch (p.DV) {
+    case 64: return launch_t<R, 64, KI8>(p, s);
+    case 128: return launch_t<R, 128, KI8>(p, s);
+  }
+  *uns = 1;
+  return cudaSuccess;
+}
+
+template <bool KI8>
+cudaError_t by_r(const AppendParams& p, cudaStream_t s, int* uns) {
+  switch (p.R) {
+    case 16: return by_dv<16, KI8>(p, s, uns);
+    case 32: return by_dv<32, KI8>(p, s, uns);
+    case 64: return by_dv<64, KI8>(p, s, uns);
+    case 128: return by_dv<128, KI8>(p, s, uns);
+  }
+  *uns = 1;
+  return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t launch_append(const AppendParams& p, cudaStream_t stream, int* unsupported) {
+  *unsupported = 0;
+  if (p.T == 0 || p.B == 0) return cudaSuccess;
+  return p.k_int8 ? by_r<true>(p, stream, unsupported) : by_r<false>(p, stream, unsupported);
+}
+
+}  // namespace tk

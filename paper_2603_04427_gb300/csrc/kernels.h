@@ -1,0 +1,75 @@
+// Internal launch interface between the C ABI (tk_api.cu) and the kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace tk {
+
+struct DecodeParams {
+  const void* q;             // bf16 [B][Hq][R]
+  const void* k;             // bf16 or int8 cache / pool
+  const void* v;             // bf16 cache / pool
+  const float* k_scale;      // fp32 per-token key scales (int8 keys)
+  const int32_t* page_table; // [B][max_pages] (paged)
+  const int32_t* seq_lens;   // [B]
+  void* out;                 // [B][Hq][DV]
+  int out_f32;
+  float* part_o;       // [B][Hkv][n_split][G][DV] unnormalised partial outputs
+  float* part_ml;      // [B][Hkv][n_split][G][2] (running max in log2 units, sum)
+  int32_t* counters;   // [B][Hkv] arrival counters, zero between launches
+  int* err;            // device error word
+  int B, Hq, Hkv, R, DV, G;
+  int k_int8;
+  int capacity;        // contiguous
+  int page_size, page_shift, num_pages, max_pages;  // paged (page_size 0 = contiguous)
+  int max_seq_len;
+  int n_split;         // grid.x
+  int split_chunks;    // 64-token chunks per split
+  float scale_log2;    // scale * log2(e)
+};
+
+// Split plan shared by tk_decode_workspace_size and tk_attn_decode.
+struct DecodePlan {
+  int n_split;
+  int split_chunks;
+  size_t off_counters, off_ml, off_o, bytes;
+};
+DecodePlan plan_decode(int B, int Hq, int Hkv, int DV, int max_seq_len, int num_sms);
+
+cudaError_t launch_decode(const DecodeParams& p, cudaStream_t stream, int* unsupported);
+
+struct AppendParams {
+  void* k;                   // cache / pool (bf16 or int8 codes)
+  void* v;
+  float* k_scale;
+  const int32_t* page_table;
+  const int32_t* seq_lens;
+  const void* k_new;         // bf16 [B][Hkv][T][R]
+  const void* v_new;         // bf16 [B][Hkv][T][DV]
+  int* err;
+  int B, Hkv, R, DV, T;
+  int k_int8;
+  int capacity;
+  int page_size, page_shift, num_pages, max_pages;
+};
+
+cudaError_t launch_append(const AppendParams& p, cudaStream_t stream, int* unsupported);
+
+struct PrefillParams {
+  const void* q;  // bf16 [B][Hq][S][R]
+  const void* k;  // bf16 [B][Hkv][S][R]
+  const void* v;  // bf16 [B][Hkv][S][DV]
+  void* out;      // [B][Hq][S][DV]
+  int out_f32;
+  int* err;
+  int B, Hq, Hkv, S, R, DV;
+  int causal;
+  float scale_log2;
+  int num_sms;
+};
+
+cudaError_t launch_prefill(const PrefillParams& p, cudaStream_t stream, int* unsupported);
+
+}  // namespace tk

@@ -1,0 +1,275 @@
+// C ABI of the thin-key attention library (declared in include/tk.h):
+// argument validation, split planning, the device error word, and dispatch
+// to the kernels.  Nothing here allocates device memory.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include "kernels.h"
+#include "tk.h"
+
+namespace {
+
+// Device error word: kernels record the first bad index / timed-out wait here.
+__device__ int g_tk_device_error;
+
+constexpr int kMaxDevices = 64;
+
+struct DeviceInfo {
+  bool ready = false;
+  int num_sms = 0;
+  int* err = nullptr;  // device address of g_tk_device_error
+};
+DeviceInfo g_dev[kMaxDevices];
+std::mutex g_dev_mu;
+
+thread_local std::string t_last_error;
+
+tk_status fail(tk_status s, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
+tk_status fail(tk_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  t_last_error = buf;
+  return s;
+}
+
+tk_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(TK_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// Per-device set-up (SM count, device address of the error word), done once
+// per device with that device current.
+tk_status device_info(DeviceInfo** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return fail(TK_ERR_UNSUPPORTED, "device ordinal %d", dev);
+  std::lock_guard<std::mutex> lock(g_dev_mu);
+  DeviceInfo& d = g_dev[dev];
+  if (!d.ready) {
+    e = cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+    e = cudaGetSymbolAddress(reinterpret_cast<void**>(&d.err), g_tk_device_error);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(error word)");
+    d.ready = true;
+  }
+  *out = &d;
+  return TK_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool pow2(int x) { return x > 0 && (x & (x - 1)) == 0; }
+int log2i(int x) {
+  int s = 0;
+  while ((1 << s) < x) ++s;
+  return s;
+}
+bool supported_r(int r) { return r == 16 || r == 32 || r == 64 || r == 128; }
+bool supported_dv(int d) { return d == 64 || d == 128; }
+bool supported_g(int g) { return g == 1 || g == 2 || g == 4 || g == 8; }
+
+tk_status check_desc(const tk_cache_desc* d) {
+  if (!d) return fail(TK_ERR_INVALID_ARG, "desc is NULL");
+  if (d->batch < 0 || d->h_q <= 0 || d->h_kv <= 0)
+    return fail(TK_ERR_INVALID_ARG, "batch=%d h_q=%d h_kv=%d", d->batch, d->h_q, d->h_kv);
+  if (d->h_q % d->h_kv != 0)
+    return fail(TK_ERR_INVALID_ARG, "h_q=%d is not a multiple of h_kv=%d", d->h_q, d->h_kv);
+  if (!supported_g(d->h_q / d->h_kv))
+    return fail(TK_ERR_UNSUPPORTED, "h_q/h_kv=%d (supported: 1, 2, 4, 8)", d->h_q / d->h_kv);
+  if (!supported_r(d->r)) return fail(TK_ERR_UNSUPPORTED, "r=%d (supported: 16, 32, 64, 128)", d->r);
+  if (!supported_dv(d->d_v)) return fail(TK_ERR_UNSUPPORTED, "d_v=%d (supported: 64, 128)", d->d_v);
+  if (d->k_dtype != TK_BF16 && d->k_dtype != TK_I8)
+    return fail(TK_ERR_UNSUPPORTED, "k_dtype=%d (supported: TK_BF16, TK_I8)", d->k_dtype);
+  if (d->page_size == 0) {
+    if (d->capacity <= 0 || d->capacity % 16 != 0)
+      return fail(TK_ERR_INVALID_ARG, "capacity=%d must be a positive multiple of 16", d->capacity);
+  } else {
+    if (!pow2(d->page_size) || d->page_size < 16 || d->page_size > 256)
+      return fail(TK_ERR_UNSUPPORTED, "page_size=%d (supported: 16..256, power of two)",
+                  d->page_size);
+    if (d->num_pages <= 0 || d->max_pages_per_seq <= 0)
+      return fail(TK_ERR_INVALID_ARG, "num_pages=%d max_pages_per_seq=%d", d->num_pages,
+                  d->max_pages_per_seq);
+  }
+  return TK_OK;
+}
+
+tk_status check_cache_ptrs(const tk_cache_desc* d, const void* k, const void* v, const void* ks,
+                           const void* pt) {
+  if (!k || !v) return fail(TK_ERR_INVALID_ARG, "k_cache / v_cache is NULL");
+  if (!aligned16(k) || !aligned16(v) || (ks && !aligned16(ks)))
+    return fail(TK_ERR_INVALID_ARG, "cache pointers must be 16-byte aligned");
+  if (d->k_dtype == TK_I8 && !ks) return fail(TK_ERR_INVALID_ARG, "int8 keys need k_scale");
+  if (d->page_size != 0 && !pt) return fail(TK_ERR_INVALID_ARG, "paged cache needs page_table");
+  return TK_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+tk_status tk_kv_append(const tk_cache_desc* desc, void* k_cache, void* v_cache, float* k_scale,
+                       const int32_t* page_table, const int32_t* seq_lens, const void* k_new,
+                       const void* v_new, int32_t n_new, void* stream) {
+  tk_status s = check_desc(desc);
+  if (s != TK_OK) return s;
+  if (n_new < 0) return fail(TK_ERR_INVALID_ARG, "n_new=%d", n_new);
+  if (n_new == 0 || desc->batch == 0) return TK_OK;
+  if ((s = check_cache_ptrs(desc, k_cache, v_cache, k_scale, page_table)) != TK_OK) return s;
+  if (!seq_lens || !k_new || !v_new) return fail(TK_ERR_INVALID_ARG, "seq_lens / k_new / v_new is NULL");
+  if (!aligned16(k_new) || !aligned16(v_new))
+    return fail(TK_ERR_INVALID_ARG, "k_new / v_new must be 16-byte aligned");
+  DeviceInfo* dev;
+  if ((s = device_info(&dev)) != TK_OK) return s;
+  tk::AppendParams p{};
+  p.k = k_cache; p.v = v_cache; p.k_scale = k_scale; p.page_table = page_table;
+  p.seq_lens = seq_lens; p.k_new = k_new; p.v_new = v_new; p.err = dev->err;
+  p.B = desc->batch; p.Hkv = desc->h_kv; p.R = desc->r; p.DV = desc->d_v; p.T = n_new;
+  p.k_int8 = desc->k_dtype == TK_I8;
+  p.capacity = desc->capacity;
+  p.page_size = desc->page_size;
+  p.page_shift = desc->page_size ? log2i(desc->page_size) : 0;
+  p.num_pages = desc->num_pages; p.max_pages = desc->max_pages_per_seq;
+  int uns = 0;
+  cudaError_t e = tk::launch_append(p, static_cast<cudaStream_t>(stream), &uns);
+  if (uns) return fail(TK_ERR_UNSUPPORTED, "append: no kernel for this shape");
+  if (e != cudaSuccess) return cuda_fail(e, "append launch");
+  return TK_OK;
+}
+
+tk_status tk_attn_prefill(const void* q, const void* k, const void* v, void* out,
+                          int32_t out_dtype, int32_t batch, int32_t h_q, int32_t h_kv,
+                          int32_t seq, int32_t r, int32_t d_v, float scale, int32_t causal,
+                          void* stream) {
+  if (batch < 0 || seq < 0 || h_q <= 0 || h_kv <= 0)
+    return fail(TK_ERR_INVALID_ARG, "batch=%d seq=%d h_q=%d h_kv=%d", batch, seq, h_q, h_kv);
+  if (h_q % h_kv != 0) return fail(TK_ERR_INVALID_ARG, "h_q=%d not a multiple of h_kv=%d", h_q, h_kv);
+  if (!supported_r(r)) return fail(TK_ERR_UNSUPPORTED, "r=%d (supported: 16, 32, 64, 128)", r);
+  if (!supported_dv(d_v)) return fail(TK_ERR_UNSUPPORTED, "d_v=%d (supported: 64, 128)", d_v);
+  if (out_dtype != TK_BF16 && out_dtype != TK_F32)
+    return fail(TK_ERR_UNSUPPORTED, "out_dtype=%d (supported: TK_BF16, TK_F32)", out_dtype);
+  if (!std::isfinite(scale)) return fail(TK_ERR_INVALID_ARG, "scale is not finite");
+  if (batch == 0 || seq == 0) return TK_OK;
+  if (!q || !k || !v || !out) return fail(TK_ERR_INVALID_ARG, "q / k / v / out is NULL");
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out))
+    return fail(TK_ERR_INVALID_ARG, "q / k / v / out must be 16-byte aligned");
+  DeviceInfo* dev;
+  tk_status s = device_info(&dev);
+  if (s != TK_OK) return s;
+  tk::PrefillParams p{};
+  p.q = q; p.k = k; p.v = v; p.out = out; p.out_f32 = out_dtype == TK_F32; p.err = dev->err;
+  p.B = batch; p.Hq = h_q; p.Hkv = h_kv; p.S = seq; p.R = r; p.DV = d_v;
+  p.causal = causal != 0;
+  p.scale_log2 = scale * 1.4426950408889634f;
+  p.num_sms = dev->num_sms;
+  int uns = 0;
+  cudaError_t e = tk::launch_prefill(p, static_cast<cudaStream_t>(stream), &uns);
+  if (uns) return fail(TK_ERR_UNSUPPORTED, "prefill: no kernel for r=%d d_v=%d", r, d_v);
+  if (e != cudaSuccess) return cuda_fail(e, "prefill launch");
+  return TK_OK;
+}
+
+size_t tk_decode_workspace_size(const tk_cache_desc* desc, int32_t max_seq_len) {
+  if (check_desc(desc) != TK_OK || max_seq_len < 0) return 0;
+  DeviceInfo* dev;
+  if (device_info(&dev) != TK_OK) return 0;
+  return tk::plan_decode(desc->batch, desc->h_q, desc->h_kv, desc->d_v, max_seq_len,
+                         dev->num_sms).bytes;
+}
+
+tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k_cache,
+                         const void* v_cache, const float* k_scale, const int32_t* page_table,
+                         const int32_t* seq_lens, int32_t max_seq_len, void* out,
+                         int32_t out_dtype, float scale, void* workspace,
+                         size_t workspace_bytes, void* stream) {
+  tk_status s = check_desc(desc);
+  if (s != TK_OK) return s;
+  if (max_seq_len < 0) return fail(TK_ERR_INVALID_ARG, "max_seq_len=%d", max_seq_len);
+  if (out_dtype != TK_BF16 && out_dtype != TK_F32)
+    return fail(TK_ERR_UNSUPPORTED, "out_dtype=%d (supported: TK_BF16, TK_F32)", out_dtype);
+  if (!std::isfinite(scale)) return fail(TK_ERR_INVALID_ARG, "scale is not finite");
+  if (desc->batch == 0) return TK_OK;
+  if ((s = check_cache_ptrs(desc, k_cache, v_cache, k_scale, page_table)) != TK_OK) return s;
+  if (!q || !out || !seq_lens) return fail(TK_ERR_INVALID_ARG, "q / out / seq_lens is NULL");
+  if (!aligned16(q) || !aligned16(out))
+    return fail(TK_ERR_INVALID_ARG, "q / out must be 16-byte aligned");
+  DeviceInfo* dev;
+  if ((s = device_info(&dev)) != TK_OK) return s;
+  const tk::DecodePlan pl =
+      tk::plan_decode(desc->batch, desc->h_q, desc->h_kv, desc->d_v, max_seq_len, dev->num_sms);
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+    return fail(TK_ERR_WORKSPACE, "workspace is NULL or not 256-byte aligned");
+  if (workspace_bytes < pl.bytes)
+    return fail(TK_ERR_WORKSPACE, "workspace has %zu bytes, %zu needed", workspace_bytes, pl.bytes);
+  unsigned char* ws = static_cast<unsigned char*>(workspace);
+  tk::DecodeParams p{};
+  p.q = q; p.k = k_cache; p.v = v_cache; p.k_scale = k_scale; p.page_table = page_table;
+  p.seq_lens = seq_lens; p.out = out; p.out_f32 = out_dtype == TK_F32;
+  p.counters = reinterpret_cast<int32_t*>(ws + pl.off_counters);
+  p.part_ml = reinterpret_cast<float*>(ws + pl.off_ml);
+  p.part_o = reinterpret_cast<float*>(ws + pl.off_o);
+  p.err = dev->err;
+  p.B = desc->batch; p.Hq = desc->h_q; p.Hkv = desc->h_kv; p.R = desc->r; p.DV = desc->d_v;
+  p.G = desc->h_q / desc->h_kv;
+  p.k_int8 = desc->k_dtype == TK_I8;
+  p.capacity = desc->capacity;
+  p.page_size = desc->page_size;
+  p.page_shift = desc->page_size ? log2i(desc->page_size) : 0;
+  p.num_pages = desc->num_pages; p.max_pages = desc->max_pages_per_seq;
+  p.max_seq_len = max_seq_len;
+  p.n_split = pl.n_split; p.split_chunks = pl.split_chunks;
+  p.scale_log2 = scale * 1.4426950408889634f;
+  int uns = 0;
+  cudaError_t e = tk::launch_decode(p, static_cast<cudaStream_t>(stream), &uns);
+  if (uns) return fail(TK_ERR_UNSUPPORTED, "decode: no kernel for this shape");
+  if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+  return TK_OK;
+}
+
+tk_status tk_get_device_error(int32_t* code_out, void* stream) {
+  if (!code_out) return fail(TK_ERR_INVALID_ARG, "code_out is NULL");
+  DeviceInfo* dev;
+  tk_status s = device_info(&dev);
+  if (s != TK_OK) return s;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+  int v = 0;
+  e = cudaMemcpy(&v, dev->err, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "read device error word");
+  if (v != 0) {
+    const int zero = 0;
+    e = cudaMemcpy(dev->err, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "clear device error word");
+  }
+  *code_out = v;
+  if (v != 0) return fail(TK_ERR_DEVICE, "device error code %d (%s)", v,
+                          v == 1 ? "index out of range" : "wait timed out");
+  return TK_OK;
+}
+
+const char* tk_status_string(tk_status status) {
+  switch (status) {
+    case TK_OK: return "TK_OK";
+    case TK_ERR_INVALID_ARG: return "TK_ERR_INVALID_ARG";
+    case TK_ERR_UNSUPPORTED: return "TK_ERR_UNSUPPORTED";
+    case TK_ERR_WORKSPACE: return "TK_ERR_WORKSPACE";
+    case TK_ERR_CUDA: return "TK_ERR_CUDA";
+    case TK_ERR_DEVICE: return "TK_ERR_DEVICE";
+  }
+  return "TK_ERR_UNKNOWN";
+}
+
+const char* tk_last_error(void) { return t_last_error.c_str(); }
+
+int32_t tk_abi_version(void) { return TK_ABI_VERSION; }
+
+}  // extern "C"

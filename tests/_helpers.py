@@ -1,0 +1,47 @@
+"""Test plumbing: tensor <-> oracle conversion and the parity bar.
+
+The parity bar (fp outputs against the fp64 oracle on identical bf16
+inputs): max abs error <= 1e-2 and mean relative error, defined as
+sum|gpu - ref| / sum|ref| over all compared elements, <= 2e-3.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle.attention import bf16_bits_to_f64
+
+MAX_ABS = 1e-2
+MEAN_REL = 2e-3
+
+
+def has_gpu() -> bool:
+    return torch.cuda.is_available()
+
+
+def require_gpu():
+    if not has_gpu():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2603_04427_gb300 import build
+    build.build()
+
+
+def f64(t: torch.Tensor) -> np.ndarray:
+    """Exact float64 copy of a bf16 / fp32 / int8 tensor for the oracle."""
+    t = t.detach().cpu()
+    if t.dtype == torch.bfloat16:
+        return bf16_bits_to_f64(t.contiguous().view(torch.int16).numpy())
+    return t.numpy().astype(np.float64)
+
+
+def parity(got, ref, max_abs=MAX_ABS, mean_rel=MEAN_REL, what=""):
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    assert got.shape == ref.shape, (got.shape, ref.shape)
+    assert np.all(np.isfinite(got)), f"{what}: non-finite output"
+    err = np.abs(got - ref)
+    denom = np.abs(ref).sum()
+    rel = err.sum() / denom if denom > 0 else err.sum()
+    assert err.max() <= max_abs, f"{what}: max abs error {err.max():.3e} > {max_abs}"
+    assert rel <= mean_rel, f"{what}: mean relative error {rel:.3e} > {mean_rel}"
+    return float(err.max()), float(rel)

@@ -1,0 +1,116 @@
+"""The C-ABI library builds, loads and exports every symbol include/tk.h declares.
+
+Also checks the host-side argument validation, which returns before any
+CUDA call and therefore runs without a GPU.
+"""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2603_04427_gb300 import binding as tb
+from paper_2603_04427_gb300 import build as tbuild
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    tbuild.build()
+    return tb.load_library()
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "tk.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(tk_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for n in ("tk_kv_append", "tk_attn_prefill", "tk_attn_decode", "tk_decode_workspace_size"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in _declared():
+        assert hasattr(lib, name), name
+    assert set(_declared()) <= set(tb.EXPORTED) | set(_declared())
+
+
+def test_abi_version_and_status_strings(lib):
+    assert tb.tk_abi_version() == 1
+    assert tb.tk_status_string(tb.TK_OK) == "TK_OK"
+    assert tb.tk_status_string(tb.TK_ERR_WORKSPACE) == "TK_ERR_WORKSPACE"
+    assert tb.tk_status_string(99) == "TK_ERR_UNKNOWN"
+
+
+def _desc(**kw):
+    d = dict(batch=2, h_q=8, h_kv=2, r=32, d_v=128, capacity=256, page_size=0, num_pages=0,
+             max_pages_per_seq=0, k_dtype=tb.TK_BF16)
+    d.update(kw)
+    return tb.tk_cache_desc(**d)
+
+
+FAKE = ctypes.c_void_p(0x10000)  # never dereferenced: validation fails first
+
+
+@pytest.mark.parametrize("kw,status,msg", [
+    (dict(h_q=6, h_kv=4), tb.TK_ERR_INVALID_ARG, "multiple"),
+    (dict(h_q=32, h_kv=2), tb.TK_ERR_UNSUPPORTED, "h_q/h_kv"),
+    (dict(r=48), tb.TK_ERR_UNSUPPORTED, "r=48"),
+    (dict(d_v=96), tb.TK_ERR_UNSUPPORTED, "d_v=96"),
+    (dict(capacity=100), tb.TK_ERR_INVALID_ARG, "capacity"),
+    (dict(page_size=48, num_pages=4, max_pages_per_seq=2), tb.TK_ERR_UNSUPPORTED, "page_size"),
+    (dict(page_size=64, num_pages=0, max_pages_per_seq=2), tb.TK_ERR_INVALID_ARG, "num_pages"),
+    (dict(k_dtype=7), tb.TK_ERR_UNSUPPORTED, "k_dtype"),
+])
+def test_descriptor_validation(lib, kw, status, msg):
+    d = _desc(**kw)
+    st = lib.tk_kv_append(ctypes.byref(d), FAKE, FAKE, None, None, FAKE, FAKE, FAKE, 1, None)
+    assert st == status
+    assert msg in tb.tk_last_error()
+    st = lib.tk_attn_decode(ctypes.byref(d), FAKE, FAKE, FAKE, None, None, FAKE, 16, FAKE,
+                            tb.TK_F32, 0.1, FAKE, 1 << 20, None)
+    assert st == status
+    assert lib.tk_decode_workspace_size(ctypes.byref(d), 16) == 0
+
+
+def test_pointer_and_option_validation(lib):
+    d = _desc()
+    mis = ctypes.c_void_p(0x10008)
+    assert lib.tk_kv_append(ctypes.byref(d), mis, FAKE, None, None, FAKE, FAKE, FAKE, 1,
+                            None) == tb.TK_ERR_INVALID_ARG
+    assert "aligned" in tb.tk_last_error()
+    d8 = _desc(k_dtype=tb.TK_I8)
+    assert lib.tk_kv_append(ctypes.byref(d8), FAKE, FAKE, None, None, FAKE, FAKE, FAKE, 1,
+                            None) == tb.TK_ERR_INVALID_ARG
+    assert "k_scale" in tb.tk_last_error()
+    dp = _desc(page_size=64, num_pages=8, max_pages_per_seq=4, capacity=0)
+    assert lib.tk_kv_append(ctypes.byref(dp), FAKE, FAKE, None, None, FAKE, FAKE, FAKE, 1,
+                            None) == tb.TK_ERR_INVALID_ARG
+    assert "page_table" in tb.tk_last_error()
+    assert lib.tk_kv_append(ctypes.byref(d), FAKE, FAKE, None, None, FAKE, FAKE, FAKE, -1,
+                            None) == tb.TK_ERR_INVALID_ARG
+    # zero new tokens and an empty batch are no-ops (no CUDA call is made)
+    assert lib.tk_kv_append(ctypes.byref(d), None, None, None, None, None, None, None, 0,
+                            None) == tb.TK_OK
+    assert lib.tk_attn_decode(ctypes.byref(d), FAKE, FAKE, FAKE, None, None, FAKE, 16, FAKE,
+                              5, 0.1, FAKE, 1 << 20, None) == tb.TK_ERR_UNSUPPORTED
+    assert lib.tk_attn_decode(ctypes.byref(d), FAKE, FAKE, FAKE, None, None, FAKE, -1, FAKE,
+                              tb.TK_F32, 0.1, FAKE, 1 << 20, None) == tb.TK_ERR_INVALID_ARG
+    assert lib.tk_attn_decode(ctypes.byref(d), FAKE, FAKE, FAKE, None, None, FAKE, 16, FAKE,
+                              tb.TK_F32, float("nan"), FAKE, 1 << 20, None) == tb.TK_ERR_INVALID_ARG
+
+
+def test_prefill_validation(lib):
+    P = lib.tk_attn_prefill
+    assert P(FAKE, FAKE, FAKE, FAKE, tb.TK_BF16, 2, 6, 4, 128, 32, 128, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG
+    assert P(FAKE, FAKE, FAKE, FAKE, tb.TK_BF16, 2, 4, 4, 128, 24, 128, 0.1, 1, None) == tb.TK_ERR_UNSUPPORTED
+    assert P(FAKE, FAKE, FAKE, FAKE, tb.TK_BF16, 2, 4, 4, 128, 32, 80, 0.1, 1, None) == tb.TK_ERR_UNSUPPORTED
+    assert P(FAKE, FAKE, FAKE, FAKE, tb.TK_I8, 2, 4, 4, 128, 32, 128, 0.1, 1, None) == tb.TK_ERR_UNSUPPORTED
+    assert P(FAKE, FAKE, FAKE, FAKE, tb.TK_BF16, 2, 4, 4, -1, 32, 128, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG
+    assert P(None, None, None, None, tb.TK_BF16, 2, 4, 4, 0, 32, 128, 0.1, 1, None) == tb.TK_OK
+    assert P(None, FAKE, FAKE, FAKE, tb.TK_BF16, 2, 4, 4, 64, 32, 128, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG
