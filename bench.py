@@ -1,0 +1,535 @@
+#!/usr/bin/env python3
+"""Benchmark of the thin-key attention hot path on GB300.
+
+Headline (one JSON line on stdout): decode KV GB/s of the Mistral-7B-shaped
+GQA decode (B=16, H_q=32, H_kv=8, r=32, d_v=128, every context 4096 tokens).
+One step = one pass of the decode path over the batch: tk_kv_append of the
+new token of every sequence (written at position 4095, so the context stays
+4096) followed by tk_attn_decode (split-KV partials and their merge, one
+launch).  The line also carries tokens/s, the roofline of the decode kernel,
+the end-to-end number through host buffers, the oracle's CPU throughput,
+SM clocks sampled during the timed region, and the other workloads
+(causal prefill TFLOP/s, paged long-context decode, int8-key decode with
+its r sweep, the GPT-2-small layer).
+
+Timing: CUDA graphs of the step sequence are replayed between two CUDA
+events on the launching stream; W untimed warm-up steps first.  The decode
+workload rotates over several cache copies whose total exceeds 4x L2, so
+no step reads cache lines left by the previous one.
+
+    python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode KV GB/s (% HBM peak), tokens/s; prefill TFLOP/s (% bf16 peak), 1 GB300"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(p))
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def source_hash(*names):
+    h = hashlib.sha256()
+    for n in names:
+        h.update(open(os.path.join(ROOT, "paper_2603_04427_gb300", "csrc", n), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, workload: str, src_hash: str):
+    """DRAM bytes per launch from a committed ncu capture, if the kernel is unchanged since."""
+    try:
+        d = json.load(open(os.path.join(ROOT, "profiles", "dram_traffic.json")))
+        e = d[kernel][workload]
+        return e["bytes_per_launch"] if e.get("source_hash") == src_hash else None
+    except Exception:
+        return None
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons while it runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,utilization.gpu,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.2)
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) >= 9:
+                rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        util = [num(r[4]) or 0.0 for r in rows]
+        loaded = [num(r[1]) for r, u in zip(rows, util) if u >= 50 and num(r[1]) is not None]
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.strip() == "Active"})
+        return {"sm_mhz": statistics.median(loaded or sm), "sm_max_mhz": max(num(r[2]) or 0 for r in rows),
+                "reasons": reasons, "samples": len(rows), "samples_under_load": len(loaded)}
+
+
+# ----------------------------------------------------------------------------- GPU side
+
+def _l2_bytes(torch):
+    try:
+        return int(torch.cuda.get_device_properties(torch.cuda.current_device()).L2_cache_size)
+    except Exception:
+        return 129 * 2 ** 20
+
+
+class DecodeRig:
+    """Caches, inputs and pre-marshalled C-ABI arguments for one decode workload.
+
+    Each copy is a complete cache plus its query / new-token / output / workspace
+    buffers; steps rotate over the copies.
+    """
+
+    def __init__(self, w, device, copies=None, k_int8=None, r=None):
+        import torch
+
+        from paper_2603_04427_gb300 import binding as tb
+        from paper_2603_04427_gb300 import inputs
+        self.tb, self.torch = tb, torch
+        self.w = w
+        self.r = r or w.r
+        self.k_int8 = w.k_int8 if k_int8 is None else k_int8
+        B, hq, hkv, dv = w.batch, w.h_q, w.h_kv, w.d_v
+        if w.seq_range:
+            self.lens = inputs.uniform_lengths(B, w.seq_range[0], w.seq_range[1], seed=w.seed)
+        else:
+            self.lens = [w.seq] * B
+        self.max_len = max(self.lens)
+        from paper_2603_04427_gb300 import cost_model as cm
+        kb = 1 if self.k_int8 else 2
+        self.kv_bytes = cm.decode_kv_bytes(self.lens, hkv, self.r, dv, k_bytes=kb,
+                                           k_scale_bytes=4 if self.k_int8 else 0)
+        self.io_bytes = cm.decode_io_bytes(B, hq, self.r, dv, out_bytes=4)
+        per_copy = self.kv_bytes
+        if copies is None:
+            copies = max(1, min(8, math.ceil(4 * _l2_bytes(torch) / per_copy)))
+        self.copies = []
+        seq_app = torch.tensor([n - 1 for n in self.lens], dtype=torch.int32, device=device)
+        seq_dec = torch.tensor(self.lens, dtype=torch.int32, device=device)
+        for c in range(copies):
+            seed = w.seed * 100 + c * 10
+            if w.page_size:
+                table, n_pages = inputs.paged_layout(self.lens, w.page_size, seed=seed)
+                cache = tb.ThinKeyCache.allocate(B, hq, hkv, self.r, dv, page_size=w.page_size,
+                                                 num_pages=n_pages, page_table=table,
+                                                 k_int8=self.k_int8, device=device)
+                self._fill_paged(cache, seed, device)
+            else:
+                cap = (self.max_len + 15) // 16 * 16
+                cache = tb.ThinKeyCache.allocate(B, hq, hkv, self.r, dv, capacity=cap,
+                                                 k_int8=self.k_int8, device=device)
+                T = self.max_len
+                kn = inputs.normal_bf16((B, hkv, T, self.r), seed + 1, device=device)
+                vn = inputs.normal_bf16((B, hkv, T, dv), seed + 2, device=device)
+                tb.tk_kv_append(cache, kn, vn, torch.zeros(B, dtype=torch.int32, device=device))
+                del kn, vn
+            q = inputs.normal_bf16((B, hq, self.r), seed + 3, device=device)
+            k1 = inputs.normal_bf16((B, hkv, 1, self.r), seed + 4, device=device)
+            v1 = inputs.normal_bf16((B, hkv, 1, dv), seed + 5, device=device)
+            out = torch.empty(B, hq, dv, dtype=torch.float32, device=device)
+            ws = tb.decode_workspace(cache.desc, self.max_len, device=device)
+            self.copies.append(dict(cache=cache, q=q, k1=k1, v1=v1, out=out, ws=ws,
+                                    seq_app=seq_app, seq_dec=seq_dec))
+        torch.cuda.synchronize()
+        if tb.tk_get_device_error() != 0:
+            raise RuntimeError("device error while building the cache")
+
+    def _fill_paged(self, cache, seed, device):
+        from paper_2603_04427_gb300 import inputs
+        torch = self.torch
+        if self.k_int8:
+            # quantise through the append kernel, one 64-token page column at a time
+            raise NotImplementedError("paged int8 rig is not used by the benchmark")
+        cache.k.copy_(inputs.normal_bf16(cache.k.shape, seed + 1, device=device))
+        cache.v.copy_(inputs.normal_bf16(cache.v.shape, seed + 2, device=device))
+
+    def step(self, i, with_append=True):
+        c = self.copies[i % len(self.copies)]
+        if with_append:
+            self.tb.tk_kv_append(c["cache"], c["k1"], c["v1"], c["seq_app"])
+        self.tb.tk_attn_decode(c["cache"], c["q"], c["seq_dec"], self.max_len, c["out"], c["ws"])
+
+
+def graph_time(torch, enqueue, steps, warmup, max_graph=256):
+    """Time exactly `steps` calls of enqueue(i) replayed from CUDA graphs; returns seconds."""
+    stream = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for i in range(warmup):
+            enqueue(i)
+    torch.cuda.synchronize()
+    G = max(1, min(steps, max_graph))
+    graphs = {}
+
+    def graph_of(n):
+        if n not in graphs:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for i in range(n):
+                    enqueue(i)
+            graphs[n] = g
+        return graphs[n]
+
+    full, rem = divmod(steps, G)
+    g_full = graph_of(G) if full else None
+    g_rem = graph_of(rem) if rem else None
+    with torch.cuda.stream(stream):   # one untimed replay uploads the graphs
+        if g_full is not None:
+            g_full.replay()
+        if g_rem is not None:
+            g_rem.replay()
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(full):
+            g_full.replay()
+        if g_rem is not None:
+            g_rem.replay()
+        t1.record(stream)
+    t1.synchronize()
+    return t0.elapsed_time(t1) / 1e3
+
+
+def measure_decode(rig, steps, warmup, with_append=True):
+    torch = rig.torch
+    sec = graph_time(torch, lambda i: rig.step(i, with_append), steps, warmup)
+    return sec / steps
+
+
+def measure_decode_e2e(rig, steps):
+    """Through host buffers: per step H2D of q and the new token's k, v from pinned
+    memory, append + decode, D2H of the output, host synchronisation."""
+    torch = rig.torch
+    c = rig.copies[0]
+    hq = c["q"].cpu().pin_memory()
+    hk = c["k1"].cpu().pin_memory()
+    hv = c["v1"].cpu().pin_memory()
+    ho = torch.empty(c["out"].shape, dtype=torch.float32).pin_memory()
+    stream = torch.cuda.Stream()
+    n = max(1, steps)
+    with torch.cuda.stream(stream):
+        for i in range(min(n, 20)):  # warm-up
+            c["q"].copy_(hq, non_blocking=True)
+            rig.step(0)
+            ho.copy_(c["out"], non_blocking=True)
+            stream.synchronize()
+        t0 = time.perf_counter()
+        for i in range(n):
+            cc = rig.copies[i % len(rig.copies)]
+            cc["q"].copy_(hq, non_blocking=True)
+            cc["k1"].copy_(hk, non_blocking=True)
+            cc["v1"].copy_(hv, non_blocking=True)
+            rig.step(i)
+            ho.copy_(cc["out"], non_blocking=True)
+            stream.synchronize()
+        dt = (time.perf_counter() - t0) / n
+    h2d = hq.numel() * 2 + hk.numel() * 2 + hv.numel() * 2
+    d2h = ho.numel() * 4
+    return dt, h2d, d2h
+
+
+def measure_prefill(w, iters, device, torch):
+    from paper_2603_04427_gb300 import binding as tb
+    from paper_2603_04427_gb300 import cost_model as cm
+    from paper_2603_04427_gb300 import inputs
+    B, hq, hkv, S, r, dv = w.batch, w.h_q, w.h_kv, w.seq, w.r, w.d_v
+    per = (B * hq * S * r + B * hkv * S * (r + dv) + B * hq * S * dv) * 2
+    copies = max(1, min(4, math.ceil(4 * _l2_bytes(torch) / per)))
+    sets = []
+    for c in range(copies):
+        s = w.seed * 100 + c * 10
+        sets.append((inputs.normal_bf16((B, hq, S, r), s + 1, device=device),
+                     inputs.normal_bf16((B, hkv, S, r), s + 2, device=device),
+                     inputs.normal_bf16((B, hkv, S, dv), s + 3, device=device),
+                     torch.empty(B, hq, S, dv, dtype=torch.bfloat16, device=device)))
+    try:
+        q, k, v, o = sets[0]
+        tb.tk_attn_prefill(q, k, v, o)
+    except tb.TkError as e:
+        if e.status == tb.TK_ERR_UNSUPPORTED:
+            return {"status": "unsupported"}
+        raise
+
+    def enq(i):
+        q, k, v, o = sets[i % len(sets)]
+        tb.tk_attn_prefill(q, k, v, o)
+
+    sec = graph_time(torch, enq, iters, 3, max_graph=16) / iters
+    flops = cm.prefill_flops(B, hq, S, r, dv, causal=True)
+    return {"ms": sec * 1e3, "tflops": flops / sec / 1e12, "flops_per_launch": flops}
+
+
+# ----------------------------------------------------------------------------- CPU oracle legs
+
+CPU_CHILD = r"""
+import json, sys, time, os
+sys.path.insert(0, os.environ["TK_ROOT"])
+import torch
+from oracle import attention as oa
+from oracle.attention import bf16_bits_to_f64
+from paper_2603_04427_gb300 import inputs, cost_model as cm
+B, hq, hkv, r, dv, L, seed, n_groups, reps, warm = [int(x) for x in sys.argv[1:11]]
+G = hq // hkv
+# a bounded sample: n_groups (sequence, kv head) groups of the workload, G query heads each
+f = lambda t: bf16_bits_to_f64(t.view(torch.int16).numpy())
+k = f(inputs.normal_bf16((1, n_groups, L, r), seed + 1))
+v = f(inputs.normal_bf16((1, n_groups, L, dv), seed + 2))
+q = f(inputs.normal_bf16((1, n_groups * G, r), seed + 3))
+for _ in range(warm):
+    oa.attention_decode(q, k, v, [L], 1.0 / r ** 0.5)
+t0 = time.perf_counter()
+for _ in range(reps):
+    oa.attention_decode(q, k, v, [L], 1.0 / r ** 0.5)
+el = time.perf_counter() - t0
+print(json.dumps({"sec": el, "reps": reps, "bytes": cm.decode_kv_bytes([L] * n_groups, 1, r, dv) * reps}))
+"""
+
+
+def cpu_oracle_decode(w, n_groups: int, reps: int, warmup: int = 1):
+    """Time `reps` oracle decodes of a sample of the workload on one host thread, in a fresh process."""
+    env = dict(os.environ, TK_ROOT=ROOT, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1",
+               MKL_NUM_THREADS="1", CUDA_VISIBLE_DEVICES="")
+    args = [str(x) for x in (w.batch, w.h_q, w.h_kv, w.r, w.d_v, w.seq, w.seed, n_groups, reps, warmup)]
+    out = subprocess.run([sys.executable, "-c", CPU_CHILD] + args, env=env, capture_output=True,
+                         text=True, timeout=900)
+    if out.returncode != 0:
+        raise RuntimeError(out.stderr[-2000:])
+    d = json.loads(out.stdout.strip().splitlines()[-1])
+    return {"value": d["bytes"] / d["sec"] / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sec": d["sec"], "reps": reps,
+            "sample": f"{n_groups} of {w.batch * w.h_kv} (sequence, kv-head) groups x "
+                      f"{w.h_q // w.h_kv} query heads at context {w.seq}, {reps} timed repetitions "
+                      f"({d['sec']:.1f} s); fp64 numpy on one thread, bf16 inputs converted before timing"}
+
+
+def run_reference(args, rank):
+    """--impl reference: the fp64 CPU oracle on the headline workload, W + K steps.
+
+    Each step is the oracle's decode over a sample of the workload's
+    (sequence, kv head) groups, sized from a short calibration so that the
+    whole run stays within about two minutes.
+    """
+    from paper_2603_04427_gb300 import workloads as wl
+    w = wl.MISTRAL_GQA_DECODE
+    if rank != 0:
+        return
+    cal = cpu_oracle_decode(w, 1, 5)
+    t_group = cal["sec"] / cal["reps"]
+    n_groups = int(max(1, min(w.batch * w.h_kv, 120.0 / (args.steps + args.warmup) / t_group)))
+    res = cpu_oracle_decode(w, n_groups, args.steps, args.warmup)
+    line = {"impl": "reference", "metric": METRIC, "value": res["value"], "unit": "GB/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": res["sec"] / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": dict(w.as_config(), sample_groups=n_groups),
+            "cpu_baseline": res,
+            "e2e": {"value": res["value"], "unit": "GB/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- main
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=200)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--headline-only", action="store_true",
+                    help="skip the secondary workloads and the CPU baseline")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank)
+        return
+
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2603_04427_gb300 import binding as tb
+    from paper_2603_04427_gb300 import cost_model as cm
+    from paper_2603_04427_gb300 import workloads as wl
+
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=device)
+    peaks, peak_src = load_peaks()
+    w = wl.MISTRAL_GQA_DECODE
+
+    rig = DecodeRig(w, device)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    clocks.start()
+    sec_step = measure_decode(rig, args.steps, args.warmup, with_append=True)
+    sec_dec = measure_decode(rig, args.steps, args.warmup, with_append=False)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if dist:
+        t = torch.tensor([sec_step, sec_dec], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        sec_step, sec_dec = float(t[0]), float(t[1])
+    n = world
+    value = n * rig.kv_bytes / sec_step / 1e9
+    e2e_dt, h2d, d2h = measure_decode_e2e(rig, min(args.steps, 5000))
+    if dist:
+        t = torch.tensor([e2e_dt], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_dt = float(t[0])
+    achieved = (rig.kv_bytes + rig.io_bytes) / sec_dec / 1e9
+    dec_hash = source_hash("decode.cu", "common.cuh")
+    line = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": n, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": sec_step * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": dict(w.as_config(), storage="bf16 K/V, fp32 accumulate, fp32 out",
+                       step="tk_kv_append(1 token) + tk_attn_decode",
+                       l2=f"rotating {len(rig.copies)} cache copies "
+                          f"({len(rig.copies) * rig.kv_bytes / 1e6:.0f} MB > 4x L2)",
+                       parallelism=f"replicas x{n}" if n > 1 else "single GPU"),
+        "tokens_per_s": n * w.batch / sec_step,
+        "kv_bytes_per_step": rig.kv_bytes,
+        "hbm_frac_of_measured_peak": value / peaks["hbm_gbs"],
+        "roofline": {"kernel": "decode_kernel<32,128,4,bf16>", "bound": "hbm",
+                     "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": achieved / peaks["hbm_gbs"], "peak_source": peak_src,
+                     "launch_us": sec_dec * 1e6,
+                     "bytes_per_launch": rig.kv_bytes + rig.io_bytes,
+                     "traffic": recorded_traffic("decode", w.name, dec_hash)},
+        "e2e": {"value": n * rig.kv_bytes / e2e_dt / 1e9, "unit": "GB/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": e2e_dt * 1e3,
+                "how": "pinned host q/k/v of the new token -> device, append + decode, "
+                       "output -> pinned host, host synchronisation every step"},
+        "gpu_launches": 2 * args.steps,
+        "clocks": clk,
+    }
+    del rig
+    torch.cuda.empty_cache()
+
+    if rank == 0 and not args.headline_only:
+        extra = {}
+        # causal prefill, B=2, H=32, S=8192, r=32, d_v=128, bf16 out
+        pw = wl.MHA7B_PREFILL
+        pf = measure_prefill(pw, 20, device, torch)
+        if "tflops" in pf:
+            pf.update(frac=pf["tflops"] / peaks["bf16_tflops"], peak=peaks["bf16_tflops"],
+                      peak_source=peak_src, bound="tensor")
+        extra[pw.name] = dict(pw.as_config(), **pf)
+        # paged long-context decode
+        pl = wl.PAGED_LONG_DECODE
+        prig = DecodeRig(pl, device, copies=1)
+        s = measure_decode(prig, 200, 20, with_append=True)
+        sd = measure_decode(prig, 200, 20, with_append=False)
+        extra[pl.name] = dict(pl.as_config(), seq_lens=prig.lens, kv_bytes=prig.kv_bytes,
+                              step_us=s * 1e6, gbs=prig.kv_bytes / s / 1e9,
+                              decode_kernel_us=sd * 1e6,
+                              decode_kernel_frac=(prig.kv_bytes + prig.io_bytes) / sd / 1e9 / peaks["hbm_gbs"])
+        del prig
+        torch.cuda.empty_cache()
+        # int8 keys, B=64, context 32768, and the r sweep (int8 and bf16 keys)
+        iw = wl.INT8_DECODE
+        sweep = []
+        for r in iw.r_sweep:
+            for k8 in (True, False):
+                rr = DecodeRig(iw, device, copies=1, k_int8=k8, r=r)
+                s = measure_decode(rr, 50, 5, with_append=True)
+                sd = measure_decode(rr, 50, 5, with_append=False)
+                sweep.append({"r": r, "k_dtype": "int8" if k8 else "bf16", "kv_bytes": rr.kv_bytes,
+                              "step_us": s * 1e6, "gbs": rr.kv_bytes / s / 1e9,
+                              "decode_kernel_us": sd * 1e6,
+                              "decode_kernel_frac": (rr.kv_bytes + rr.io_bytes) / sd / 1e9 / peaks["hbm_gbs"]})
+                del rr
+                torch.cuda.empty_cache()
+        extra[iw.name] = dict(iw.as_config(), sweep=sweep)
+        line["workloads"] = extra
+        try:
+            cal = cpu_oracle_decode(w, 1, 5)
+            reps = max(1, int(10.0 / (cal["sec"] / cal["reps"] * 16)))
+            line["cpu_baseline"] = cpu_oracle_decode(w, 16, reps) if n == 1 else None
+        except Exception as e:  # reported, not fatal
+            line["cpu_baseline"] = {"error": str(e)[-300:]}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -128,7 +128,7 @@ tk_status tk_kv_append(const tk_cache_desc* desc, void* k_cache, void* v_cache, 
  *   v   : device bf16 [batch][h_kv][seq][d_v]
  *   out : device [batch][h_q][seq][d_v], bf16 (out_dtype TK_BF16, round to
  *         nearest even) or fp32 (TK_F32)
- *   scale: multiplies q.k (the paper uses 1/sqrt(r))
+ *   scale: multiplies q.k (the paper uses 1/sqrt(r)); must be > 0
  *   causal: nonzero = query i attends to keys 0..i (top-left aligned);
  *           zero = every query attends to all seq keys.
  * Shapes: r in {16, 32, 64, 128}, d_v in {64, 128}, h_q % h_kv == 0,

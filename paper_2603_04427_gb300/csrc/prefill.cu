@@ -1,9 +1,491 @@
-// Causal prefill attention (tcgen05 / TMEM / TMA): not built yet.
+// Causal (or full) prefill attention with thin keys on the 5th-generation
+// tensor cores: tcgen05.mma with accumulators in tensor memory (TMEM),
+// operands staged in shared memory by TMA.
+//
+// Paper: Section 2.1, Eqs. 1-4 (softmax(Q K^T * scale) V with r-wide Q, K and
+// d_v-wide V); Appendix E (prefill is compute-bound; thin keys cut the Q K^T
+// work by d_head / r).
+//
+// One CTA computes one 128-row query tile of one (sequence, query head):
+//   warp 4 (one lane): TMA loads of the Q tile (once) and of 128-row K and V
+//     tiles into a 2-stage shared-memory ring ("full" / "empty" mbarriers).
+//   warp 5 (one lane): issues, per kv tile j,
+//       S_j = Q K_j^T            (M=128, N=128, K=r; bf16 in, fp32 in TMEM)
+//       O  += P_j V_j            (M=128, N=d_v, K=128; P_j read from TMEM)
+//     and signals completion with tcgen05.commit onto mbarriers.
+//   warps 0-3 (thread i owns query row i = TMEM lane i): read S_j from
+//     TMEM, apply the causal / length mask, keep the running max m and sum l
+//     (log2 domain), write P_j = exp2(S_j * scale*log2e - m) as bf16 into the
+//     first 64 TMEM columns of S_j, and at the end write O / l.
+// The running max is updated lazily: O and l are rescaled only when a tile's
+// maximum exceeds the max in use by more than 8 (a factor 256), so the
+// weights stay <= 256 and the result is unchanged (O / l uses one consistent
+// max).  Two CTAs share an SM (256 TMEM columns each), so one CTA's softmax
+// overlaps the other's matrix products.
+//
+// TMEM columns per CTA: [0, 128) S (fp32; its first 64 columns hold P as
+// packed bf16 pairs), [128, 128 + d_v) O (fp32).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "common.cuh"
 #include "kernels.h"
 
 namespace tk {
-cudaError_t launch_prefill(const PrefillParams&, cudaStream_t, int* unsupported) {
+namespace {
+
+constexpr int kBM = 128;          // query rows per tile
+constexpr int kBN = 128;          // keys per kv tile
+constexpr int kStages = 2;
+constexpr int kThreads = 192;     // 4 softmax warps, 1 TMA warp, 1 MMA warp
+constexpr int kTmemCols = 256;
+constexpr float kRescaleThreshold = 8.0f;  // log2 units
+
+// ---------------------------------------------------------------- tcgen05 helpers
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_addr(dst_smem)),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_addr(bar))
+      : "memory");
+}
+// D(tmem) (+)= A(smem desc) * B(smem desc)
+__device__ __forceinline__ void mma_ss(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc,
+                                       uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// D(tmem) (+)= A(tmem) * B(smem desc)
+__device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a, uint64_t b, uint32_t idesc,
+                                       uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
+      "r"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+#define TK_R8(i) "=r"(v[i]), "=r"(v[i + 1]), "=r"(v[i + 2]), "=r"(v[i + 3]), "=r"(v[i + 4]), \
+                 "=r"(v[i + 5]), "=r"(v[i + 6]), "=r"(v[i + 7])
+#define TK_W8(i) "r"(v[i]), "r"(v[i + 1]), "r"(v[i + 2]), "r"(v[i + 3]), "r"(v[i + 4]), \
+                 "r"(v[i + 5]), "r"(v[i + 6]), "r"(v[i + 7])
+
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* v) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, "
+      "%28, %29, %30, %31}, [%32];"
+      : TK_R8(0), TK_R8(8), TK_R8(16), TK_R8(24)
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, "
+      "%28, %29, %30, %31, %32};" ::"r"(taddr),
+      TK_W8(0), TK_W8(8), TK_W8(16), TK_W8(24)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// 3-D TMA tile load into shared memory, completion on `bar`.
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z,
+                                            uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_addr(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void prefetch_map(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+// Shared-memory matrix descriptor (tcgen05 format): start address, leading and
+// stride byte offsets (all >> 4), descriptor version 1, swizzle layout code.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo,
+                                              uint32_t layout) {
+  return static_cast<uint64_t>((saddr >> 4) & 0x3FFFu) |
+         (static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16) |
+         (static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46) |
+         (static_cast<uint64_t>(layout & 7u) << 61);
+}
+
+// Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, A K-major.
+constexpr uint32_t instr_desc(int M, int N, bool b_mn_major) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
+         (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+template <int R, int DV>
+struct PCfg {
+  // Q / K rows are r bf16 = 2r bytes: swizzle span = min(2r, 128) bytes; a row
+  // wider than 128 bytes is loaded as 128-byte-wide boxes.
+  static constexpr int QK_SW = (2 * R < 128) ? 2 * R : 128;
+  static constexpr int QK_BOX = QK_SW / 2;           // elements per box row
+  static constexpr int QK_NBOX = (2 * R) / QK_SW;    // boxes per tile
+  static constexpr int QK_BOXB = kBM * QK_SW;        // bytes per box
+  static constexpr uint32_t QK_LAYOUT = QK_SW == 32 ? 6u : (QK_SW == 64 ? 4u : 2u);
+  static constexpr int KSTEP_PER_BOX = QK_SW / 32;   // 16-element K steps per box
+  static constexpr int QB = kBM * R * 2;
+  static constexpr int KB = kBN * R * 2;
+  static constexpr int VB = kBN * DV * 2;
+  static constexpr int V_NBOX = DV / 64;             // 128-byte-wide boxes of V
+  static constexpr int V_BOXB = kBN * 128;
+  static constexpr int OFF_Q = 0;
+  static constexpr int OFF_K = (QB + 1023) / 1024 * 1024;
+  static constexpr int STAGE = (KB + 1023) / 1024 * 1024 + VB;
+  static constexpr int OFF_BAR = OFF_K + kStages * STAGE;
+  static constexpr int SMEM_USED = OFF_BAR + 256;
+  static constexpr int SMEM = SMEM_USED + 1024;      // + slack to align the base to 1 KB
+  static constexpr uint32_t IDESC_S = instr_desc(kBM, kBN, false);
+  static constexpr uint32_t IDESC_O = instr_desc(kBM, DV, true);
+};
+
+struct Maps {
+  CUtensorMap q, k, v;
+};
+
+template <int R, int DV>
+__global__ void __launch_bounds__(kThreads, 2)
+prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
+  using C = PCfg<R, DV>;
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
+  uint64_t* q_full = bars + 0;
+  uint64_t* k_full = bars + 1;                  // [kStages]
+  uint64_t* v_full = k_full + kStages;          // [kStages]
+  uint64_t* kv_empty = v_full + kStages;        // [kStages]
+  uint64_t* s_full = kv_empty + kStages;
+  uint64_t* p_full = s_full + 1;
+  uint64_t* o_full = p_full + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_full + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int n_qt = (p.S + kBM - 1) / kBM;
+  const int BH = p.B * p.Hq;
+  const int qt = n_qt - 1 - static_cast<int>(blockIdx.x / BH);  // heaviest tiles first
+  const int bh = static_cast<int>(blockIdx.x % BH);
+  const int b = bh / p.Hq, h = bh % p.Hq;
+  const int kv_plane = b * p.Hkv + h / (p.Hq / p.Hkv);
+  const int n_kv_all = (p.S + kBN - 1) / kBN;
+  const int n_kv = p.causal ? min(n_kv_all, ((qt + 1) * kBM + kBN - 1) / kBN) : n_kv_all;
+
+  if (tid == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&v_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+    }
+    mbar_init(s_full, 1);
+    mbar_init(p_full, 128);
+    mbar_init(o_full, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 4) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t tS = tmem, tO = tmem + 128;
+
+  if (warp == 4) {
+    // ------------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      prefetch_map(&maps.q);
+      prefetch_map(&maps.k);
+      prefetch_map(&maps.v);
+      mbar_arrive_expect_tx(q_full, C::QB);
+      for (int i = 0; i < C::QK_NBOX; ++i)
+        tma_load_3d(smem + C::OFF_Q + i * C::QK_BOXB, &maps.q, i * C::QK_BOX, qt * kBM, bh, q_full);
+      for (int j = 0; j < n_kv; ++j) {
+        const int st = j % kStages;
+        if (j >= kStages && !mbar_wait(&kv_empty[st], ((j / kStages) - 1) & 1, p.err)) {
+          *abort_flag = 1;
+          break;
+        }
+        unsigned char* sk = smem + C::OFF_K + st * C::STAGE;
+        unsigned char* sv = sk + (C::KB + 1023) / 1024 * 1024;
+        mbar_arrive_expect_tx(&k_full[st], C::KB);
+        for (int i = 0; i < C::QK_NBOX; ++i)
+          tma_load_3d(sk + i * C::QK_BOXB, &maps.k, i * C::QK_BOX, j * kBN, kv_plane, &k_full[st]);
+        mbar_arrive_expect_tx(&v_full[st], C::VB);
+        for (int i = 0; i < C::V_NBOX; ++i)
+          tma_load_3d(sv + i * C::V_BOXB, &maps.v, i * 64, j * kBN, kv_plane, &v_full[st]);
+      }
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      bool ok = mbar_wait(q_full, 0, p.err);
+      const uint32_t q_base = smem_addr(smem + C::OFF_Q);
+      for (int j = 0; ok && j < n_kv; ++j) {
+        const int st = j % kStages;
+        const uint32_t ph = (j / kStages) & 1;
+        const uint32_t k_base = smem_addr(smem + C::OFF_K + st * C::STAGE);
+        const uint32_t v_base = k_base + (C::KB + 1023) / 1024 * 1024;
+        if (!(ok = mbar_wait(&k_full[st], ph, p.err))) break;
+        tc_fence_after();
+#pragma unroll
+        for (int k = 0; k < R / 16; ++k) {
+          const uint32_t off = (k / C::KSTEP_PER_BOX) * C::QK_BOXB + (k % C::KSTEP_PER_BOX) * 32;
+          mma_ss(tS, smem_desc(q_base + off, 16, 8 * C::QK_SW, C::QK_LAYOUT),
+                 smem_desc(k_base + off, 16, 8 * C::QK_SW, C::QK_LAYOUT), C::IDESC_S, k > 0);
+        }
+        tc_commit(s_full);
+        if (!(ok = mbar_wait(p_full, j & 1, p.err))) break;
+        tc_fence_after();
+        if (!(ok = mbar_wait(&v_full[st], ph, p.err))) break;
+#pragma unroll
+        for (int k = 0; k < kBN / 16; ++k)
+          mma_ts(tO, tS + 8 * k, smem_desc(v_base + k * 16 * 128, C::V_BOXB, 1024, 2u),
+                 C::IDESC_O, (j > 0 || k > 0) ? 1u : 0u);
+        tc_commit(&kv_empty[st]);
+      }
+      if (ok) tc_commit(o_full);
+      else *abort_flag = 1;
+    }
+  } else {
+    // ------------------------------------------------------------------ softmax warps
+    const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+    const int row = qt * kBM + tid;            // query position of this thread
+    const float sl2 = p.scale_log2;
+    float m_used = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < n_kv; ++j) {
+      ok = mbar_wait(s_full, j & 1, p.err);
+      if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
+      tc_fence_after();
+      const int kv0 = j * kBN;
+      const bool masked = (p.causal && kv0 + kBN - 1 > qt * kBM) || (kv0 + kBN > p.S);
+      const int lim = min(p.S - kv0, p.causal ? row - kv0 + 1 : kBN);  // visible columns
+      // pass 1: tile max of the raw scores
+      float mx = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint32_t v[32];
+        tmem_ld32(tS + lane_off + 32 * c, v);
+        tmem_wait_ld();
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float s = __uint_as_float(v[i]);
+          if (!masked || 32 * c + i < lim) mx = fmaxf(mx, s);
+        }
+      }
+      const float mt = mx * sl2;
+      const bool resc = mt > m_used + kRescaleThreshold;
+      float alpha = 1.f;
+      if (resc) {
+        alpha = fast_exp2(m_used - mt);   // 0 on the first tile
+        m_used = mt;
+      }
+      l *= alpha;
+      if (j > 0 && __any_sync(0xffffffffu, resc)) {
+        // O *= alpha; the previous P V product is complete (the S_j commit covers it)
+#pragma unroll
+        for (int c = 0; c < DV / 32; ++c) {
+          uint32_t v[32];
+          tmem_ld32(tO + lane_off + 32 * c, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
+          tmem_st32(tO + lane_off + 32 * c, v);
+        }
+      }
+      // pass 2: P = exp2(s * scale log2e - m) as bf16 pairs into TMEM columns [0, 64)
+      const float neg_m = -m_used;
+      float lsum0 = 0.f, lsum1 = 0.f;
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        uint32_t pk[32];
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          uint32_t v[32];
+          tmem_ld32(tS + lane_off + 64 * c + 32 * half, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; i += 2) {
+            const int col = 64 * c + 32 * half + i;
+            float p0 = fast_exp2(fmaf(__uint_as_float(v[i]), sl2, neg_m));
+            float p1 = fast_exp2(fmaf(__uint_as_float(v[i + 1]), sl2, neg_m));
+            if (masked) {
+              if (col >= lim) p0 = 0.f;
+              if (col + 1 >= lim) p1 = 0.f;
+            }
+            lsum0 += p0;
+            lsum1 += p1;
+            __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);  // low half = column col
+            pk[16 * half + i / 2] = *reinterpret_cast<uint32_t*>(&pr);
+          }
+        }
+        tmem_st32(tS + lane_off + 32 * c, pk);
+      }
+      l += lsum0 + lsum1;
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(p_full);
+    }
+    // epilogue: out = O / l
+    if (ok) ok = mbar_wait(o_full, 0, p.err);
+    if (__all_sync(0xffffffffu, ok)) {
+      tc_fence_after();
+      const float inv = 1.f / l;
+      const bool store = row < p.S;
+      const size_t obase = (static_cast<size_t>(bh) * p.S + row) * DV;
+#pragma unroll
+      for (int c = 0; c < DV / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld32(tO + lane_off + 32 * c, v);
+        tmem_wait_ld();
+        if (store) {
+          if (p.out_f32) {
+            float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.out) + obase + 32 * c);
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+              dst[i] = make_float4(__uint_as_float(v[4 * i]) * inv, __uint_as_float(v[4 * i + 1]) * inv,
+                                   __uint_as_float(v[4 * i + 2]) * inv, __uint_as_float(v[4 * i + 3]) * inv);
+          } else {
+            uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(p.out) + obase + 32 * c);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              uint32_t w[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                __nv_bfloat162 pr = __floats2bfloat162_rn(__uint_as_float(v[8 * i + 2 * e]) * inv,
+                                                          __uint_as_float(v[8 * i + 2 * e + 1]) * inv);
+                w[e] = *reinterpret_cast<uint32_t*>(&pr);
+              }
+              dst[i] = make_uint4(w[0], w[1], w[2], w[3]);
+            }
+          }
+        }
+      }
+    } else {
+      *abort_flag = 1;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 4) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ---------------------------------------------------------------- host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+// 3-D bf16 map over [planes][rows][inner] with a (box_inner x 128 x 1) box.
+bool make_map(CUtensorMap* m, const void* base, int inner, int rows, int planes, int box_inner,
+              int swizzle_bytes) {
+  auto enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows),
+                        static_cast<cuuint64_t>(planes)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(inner) * 2,
+                           static_cast<cuuint64_t>(inner) * rows * 2};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(box_inner), 128, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUtensorMapSwizzle sw = swizzle_bytes == 32   ? CU_TENSOR_MAP_SWIZZLE_32B
+                          : swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                : CU_TENSOR_MAP_SWIZZLE_128B;
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int R, int DV>
+cudaError_t launch_t(const PrefillParams& p, cudaStream_t stream) {
+  using C = PCfg<R, DV>;
+  Maps maps;
+  if (!make_map(&maps.q, p.q, R, p.S, p.B * p.Hq, C::QK_BOX, C::QK_SW) ||
+      !make_map(&maps.k, p.k, R, p.S, p.B * p.Hkv, C::QK_BOX, C::QK_SW) ||
+      !make_map(&maps.v, p.v, DV, p.S, p.B * p.Hkv, 64, 128))
+    return cudaErrorInvalidValue;
+  auto kern = prefill_kernel<R, DV>;
+  // More than a third of the SM's shared memory per CTA keeps it at <= 2 CTAs
+  // per SM, so two 256-column TMEM allocations always fit.
+  const int smem = C::SMEM > 80 * 1024 ? C::SMEM : 80 * 1024;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  const long n_qt = (p.S + kBM - 1) / kBM;
+  const long grid = n_qt * p.B * p.Hq;
+  if (grid > 0x7fffffffL) return cudaErrorInvalidConfiguration;
+  kern<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(maps, p);
+  return cudaGetLastError();
+}
+
+template <int R>
+cudaError_t by_dv(const PrefillParams& p, cudaStream_t s, int* uns) {
+  switch (p.DV) {
+    case 64: return launch_t<R, 64>(p, s);
+    case 128: return launch_t<R, 128>(p, s);
+  }
+  *uns = 1;
+  return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t launch_prefill(const PrefillParams& p, cudaStream_t stream, int* unsupported) {
+  *unsupported = 0;
+  switch (p.R) {
+    case 16: return by_dv<16>(p, stream, unsupported);
+    case 32: return by_dv<32>(p, stream, unsupported);
+    case 64: return by_dv<64>(p, stream, unsupported);
+    case 128: return by_dv<128>(p, stream, unsupported);
+  }
   *unsupported = 1;
   return cudaSuccess;
 }
+
 }  // namespace tk

@@ -156,7 +156,8 @@ tk_status tk_attn_prefill(const void* q, const void* k, const void* v, void* out
   if (!supported_dv(d_v)) return fail(TK_ERR_UNSUPPORTED, "d_v=%d (supported: 64, 128)", d_v);
   if (out_dtype != TK_BF16 && out_dtype != TK_F32)
     return fail(TK_ERR_UNSUPPORTED, "out_dtype=%d (supported: TK_BF16, TK_F32)", out_dtype);
-  if (!std::isfinite(scale)) return fail(TK_ERR_INVALID_ARG, "scale is not finite");
+  if (!std::isfinite(scale) || !(scale > 0.f))
+    return fail(TK_ERR_INVALID_ARG, "prefill scale must be finite and positive");
   if (batch == 0 || seq == 0) return TK_OK;
   if (!q || !k || !v || !out) return fail(TK_ERR_INVALID_ARG, "q / k / v / out is NULL");
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out))
