@@ -93,14 +93,32 @@ __device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a, uint64_t b, uint3
 #define TK_W8(i) "r"(v[i]), "r"(v[i + 1]), "r"(v[i + 2]), "r"(v[i + 3]), "r"(v[i + 4]), \
                  "r"(v[i + 5]), "r"(v[i + 6]), "r"(v[i + 7])
 
-// 32 consecutive fp32 columns of this thread's TMEM lane.
+// 32 consecutive 32-bit columns of this thread's TMEM lane.  The load and its
+// wait are one asm statement: tcgen05.ld fills the registers asynchronously,
+// so no use of them may be scheduled before tcgen05.wait::ld.
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* v) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
       "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, "
-      "%28, %29, %30, %31}, [%32];"
+      "%28, %29, %30, %31}, [%32];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
       : TK_R8(0), TK_R8(8), TK_R8(16), TK_R8(24)
-      : "r"(taddr));
+      : "r"(taddr)
+      : "memory");
+}
+// 64 consecutive 32-bit columns (two loads, one wait).
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, uint32_t* v) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, "
+      "%28, %29, %30, %31}, [%64];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%32, %33, %34, %35, %36, %37, %38, %39, %40, "
+      "%41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, "
+      "%58, %59, %60, %61, %62, %63}, [%65];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : TK_R8(0), TK_R8(8), TK_R8(16), TK_R8(24), TK_R8(32), TK_R8(40), TK_R8(48), TK_R8(56)
+      : "r"(taddr), "r"(taddr + 32)
+      : "memory");
 }
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* v) {
   asm volatile(
@@ -109,9 +127,6 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* v) {
       "%28, %29, %30, %31, %32};" ::"r"(taddr),
       TK_W8(0), TK_W8(8), TK_W8(16), TK_W8(24)
       : "memory");
-}
-__device__ __forceinline__ void tmem_wait_ld() {
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 __device__ __forceinline__ void tmem_wait_st() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
@@ -299,14 +314,13 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       // pass 1: tile max of the raw scores
       float mx = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        uint32_t v[32];
-        tmem_ld32(tS + lane_off + 32 * c, v);
-        tmem_wait_ld();
+      for (int c = 0; c < 2; ++c) {
+        uint32_t v[64];
+        tmem_ld64(tS + lane_off + 64 * c, v);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
+        for (int i = 0; i < 64; ++i) {
           const float s = __uint_as_float(v[i]);
-          if (!masked || 32 * c + i < lim) mx = fmaxf(mx, s);
+          if (!masked || 64 * c + i < lim) mx = fmaxf(mx, s);
         }
       }
       const float mt = mx * sl2;
@@ -323,7 +337,6 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
         for (int c = 0; c < DV / 32; ++c) {
           uint32_t v[32];
           tmem_ld32(tO + lane_off + 32 * c, v);
-          tmem_wait_ld();
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
           tmem_st32(tO + lane_off + 32 * c, v);
@@ -335,25 +348,21 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
         uint32_t pk[32];
+        uint32_t v[64];
+        tmem_ld64(tS + lane_off + 64 * c, v);
 #pragma unroll
-        for (int half = 0; half < 2; ++half) {
-          uint32_t v[32];
-          tmem_ld32(tS + lane_off + 64 * c + 32 * half, v);
-          tmem_wait_ld();
-#pragma unroll
-          for (int i = 0; i < 32; i += 2) {
-            const int col = 64 * c + 32 * half + i;
-            float p0 = fast_exp2(fmaf(__uint_as_float(v[i]), sl2, neg_m));
-            float p1 = fast_exp2(fmaf(__uint_as_float(v[i + 1]), sl2, neg_m));
-            if (masked) {
-              if (col >= lim) p0 = 0.f;
-              if (col + 1 >= lim) p1 = 0.f;
-            }
-            lsum0 += p0;
-            lsum1 += p1;
-            __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);  // low half = column col
-            pk[16 * half + i / 2] = *reinterpret_cast<uint32_t*>(&pr);
+        for (int i = 0; i < 64; i += 2) {
+          const int col = 64 * c + i;
+          float p0 = fast_exp2(fmaf(__uint_as_float(v[i]), sl2, neg_m));
+          float p1 = fast_exp2(fmaf(__uint_as_float(v[i + 1]), sl2, neg_m));
+          if (masked) {
+            if (col >= lim) p0 = 0.f;
+            if (col + 1 >= lim) p1 = 0.f;
           }
+          lsum0 += p0;
+          lsum1 += p1;
+          __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);  // low half = column col
+          pk[i / 2] = *reinterpret_cast<uint32_t*>(&pr);
         }
         tmem_st32(tS + lane_off + 32 * c, pk);
       }
@@ -373,7 +382,6 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       for (int c = 0; c < DV / 32; ++c) {
         uint32_t v[32];
         tmem_ld32(tO + lane_off + 32 * c, v);
-        tmem_wait_ld();
         if (store) {
           if (p.out_f32) {
             float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.out) + obase + 32 * c);

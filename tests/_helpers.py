@@ -3,6 +3,12 @@
 The parity bar (fp outputs against the fp64 oracle on identical bf16
 inputs): max abs error <= 1e-2 and mean relative error, defined as
 sum|gpu - ref| / sum|ref| over all compared elements, <= 2e-3.
+
+For kernels whose output is bf16, both sides take the final rounding in
+the same precision: the oracle's fp64 result is rounded to bf16 (round to
+nearest even) before the comparison.  Against the unrounded oracle the
+rounding of a correct result alone already costs about 1.4e-3 of the 2e-3
+budget.
 """
 
 import numpy as np
@@ -32,6 +38,12 @@ def f64(t: torch.Tensor) -> np.ndarray:
     if t.dtype == torch.bfloat16:
         return bf16_bits_to_f64(t.contiguous().view(torch.int16).numpy())
     return t.numpy().astype(np.float64)
+
+
+def round_bf16(x) -> np.ndarray:
+    """fp64 values rounded to bf16 (round to nearest even), back as fp64."""
+    t = torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32)).to(torch.bfloat16)
+    return t.to(torch.float64).numpy()
 
 
 def parity(got, ref, max_abs=MAX_ABS, mean_rel=MEAN_REL, what=""):
