@@ -168,6 +168,35 @@ tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k
                          int32_t out_dtype, float scale, void* workspace,
                          size_t workspace_bytes, void* stream);
 
+/* Size of the fixed device scratch array used by tk_attn_decode_noalloc. */
+#define TK_DECODE_NOALLOC_SCRATCH_BYTES (8u << 20)
+
+/* tk_attn_decode without a workspace argument, for callers that cannot
+ * allocate device memory: runtimes whose device memory is entirely held by
+ * their own pool and that forbid cudaMalloc on the decode path (it
+ * synchronises the device and can fail), plugin hosts that pass a plugin only
+ * its inputs and outputs, and real-time loops that must not touch an
+ * allocator between steps.  The paper has no counterpart; this is an
+ * interface convenience around the same decode kernel.
+ *   Arguments, layouts, results and errors are those of tk_attn_decode.
+ *   The split partials and arrival counters live in one static device array
+ *   of TK_DECODE_NOALLOC_SCRATCH_BYTES (8 MiB) in this library, which every
+ *   GPU that loads the library keeps until the process exits.  A shape whose
+ *   tk_decode_workspace_size exceeds it is rejected with TK_ERR_WORKSPACE
+ *   (tk_last_error gives both sizes) before anything is launched.
+ *   No device memory is allocated or freed.  The first call on each device
+ *   looks up the array's device address (with that device current) and
+ *   caches it; make that first call before any stream capture.  Each call
+ *   clears the counters with one cudaMemsetAsync on `stream`.
+ *   All calls on a device share the array and it keeps the last call's
+ *   contents: calls that may overlap on the GPU (different streams without
+ *   ordering between them) race and give wrong results.                   */
+tk_status tk_attn_decode_noalloc(const tk_cache_desc* desc, const void* q, const void* k_cache,
+                                 const void* v_cache, const float* k_scale,
+                                 const int32_t* page_table, const int32_t* seq_lens,
+                                 int32_t max_seq_len, void* out, int32_t out_dtype, float scale,
+                                 void* stream);
+
 /* Synchronise `stream`, then read and clear the device error word of the
  * current device: *code_out = 0 if no kernel recorded an error since the
  * last call, else a nonzero code (1 = index out of range, 2 = a wait timed

@@ -22,7 +22,8 @@ TK_BF16, TK_F32, TK_I8 = 0, 1, 2
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtk.so")
 
 EXPORTED = ("tk_kv_append", "tk_attn_prefill", "tk_decode_workspace_size", "tk_attn_decode",
-            "tk_get_device_error", "tk_status_string", "tk_last_error", "tk_abi_version")
+            "tk_attn_decode_noalloc", "tk_get_device_error", "tk_status_string", "tk_last_error",
+            "tk_abi_version")
 
 
 class TkError(RuntimeError):
@@ -56,6 +57,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tk_attn_prefill": (i32, [vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, i32, vp]),
         "tk_decode_workspace_size": (sz, [dp, i32]),
         "tk_attn_decode": (i32, [dp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp, sz, vp]),
+        "tk_attn_decode_noalloc": (i32, [dp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp]),
         "tk_get_device_error": (i32, [ctypes.POINTER(i32), vp]),
         "tk_status_string": (ctypes.c_char_p, [i32]),
         "tk_last_error": (ctypes.c_char_p, []),
@@ -223,6 +225,32 @@ def tk_attn_prefill(q, k, v, out, scale: float | None = None, causal: bool = Tru
                              TK_F32 if out.dtype == torch.float32 else TK_BF16,
                              B, hq, hkv, S, r, dv, scale, 1 if causal else 0, _stream(stream)),
            "tk_attn_prefill")
+    return out
+
+
+def tk_attn_decode_noalloc(cache: ThinKeyCache, q, seq_lens, max_seq_len: int, out,
+                           scale: float | None = None, stream=None):
+    """tk_attn_decode without a workspace: uses the library's fixed device scratch.
+
+    For callers that cannot allocate device memory.  Calls that may overlap on
+    the GPU share the scratch and race; see include/tk.h.
+    """
+    d = cache.desc
+    dev = cache.k.device
+    _need(q, torch.bfloat16, "q", dev)
+    _need(seq_lens, torch.int32, "seq_lens", dev)
+    if out.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("out must be float32 or bfloat16")
+    _need(out, out.dtype, "out", dev)
+    if tuple(q.shape) != (d.batch, d.h_q, d.r) or tuple(out.shape) != (d.batch, d.h_q, d.d_v):
+        raise ValueError(f"q {tuple(q.shape)} / out {tuple(out.shape)} do not match the cache")
+    scale = 1.0 / math.sqrt(d.r) if scale is None else float(scale)
+    L = load_library()
+    _check(L.tk_attn_decode_noalloc(ctypes.byref(d), _ptr(q), _ptr(cache.k), _ptr(cache.v),
+                                    _ptr(cache.k_scale), _ptr(cache.page_table), _ptr(seq_lens),
+                                    int(max_seq_len), _ptr(out),
+                                    TK_F32 if out.dtype == torch.float32 else TK_BF16, scale,
+                                    _stream(stream)), "tk_attn_decode_noalloc")
     return out
 
 
