@@ -294,6 +294,7 @@ def measure_decode_e2e(rig, steps):
 
 
 def measure_prefill(w, iters, device, torch):
+    """Causal prefill, bf16 output, rotating input copies (> 4x L2 in total)."""
     from paper_2603_04427_gb300 import binding as tb
     from paper_2603_04427_gb300 import cost_model as cm
     from paper_2603_04427_gb300 import inputs
@@ -322,6 +323,40 @@ def measure_prefill(w, iters, device, torch):
     sec = graph_time(torch, enq, iters, 3, max_graph=16) / iters
     flops = cm.prefill_flops(B, hq, S, r, dv, causal=True)
     return {"ms": sec * 1e3, "tflops": flops / sec / 1e12, "flops_per_launch": flops}
+
+
+def measure_gpt2_layer(w, iters, device, torch):
+    """GPT-2-small layer: causal prefill of S tokens (fp32 out), append of the
+    prompt's keys/values, then `decode_steps` x (append 1 token + decode)."""
+    from paper_2603_04427_gb300 import binding as tb
+    from paper_2603_04427_gb300 import cost_model as cm
+    from paper_2603_04427_gb300 import inputs
+    B, H, r, dv, S, T = w.batch, w.h_q, w.r, w.d_v, w.seq, w.decode_steps
+    q = inputs.normal_bf16((B, H, S, r), w.seed + 1, device=device)
+    k = inputs.normal_bf16((B, H, S, r), w.seed + 2, device=device)
+    v = inputs.normal_bf16((B, H, S, dv), w.seed + 3, device=device)
+    pre = torch.empty(B, H, S, dv, dtype=torch.float32, device=device)
+    cache = tb.ThinKeyCache.allocate(B, H, H, r, dv, capacity=S + T, device=device)
+    qd = inputs.normal_bf16((T, B, H, r), w.seed + 4, device=device)
+    kd = inputs.normal_bf16((T, B, H, 1, r), w.seed + 5, device=device)
+    vd = inputs.normal_bf16((T, B, H, 1, dv), w.seed + 6, device=device)
+    out = torch.empty(T, B, H, dv, dtype=torch.float32, device=device)
+    ws = tb.decode_workspace(cache.desc, S + T, device=device)
+    zero = torch.zeros(B, dtype=torch.int32, device=device)
+    lens = [torch.full((B,), S + t, dtype=torch.int32, device=device) for t in range(T + 1)]
+
+    def layer(_):
+        tb.tk_attn_prefill(q, k, v, pre)
+        tb.tk_kv_append(cache, k, v, zero)
+        for t in range(T):
+            tb.tk_kv_append(cache, kd[t], vd[t], lens[t])
+            tb.tk_attn_decode(cache, qd[t], lens[t + 1], S + T, out[t], ws)
+
+    sec = graph_time(torch, layer, iters, 3, max_graph=4) / iters
+    flops = cm.prefill_flops(B, H, S, r, dv)
+    kv = sum(cm.decode_kv_bytes([S + t + 1] * B, H, r, dv) for t in range(T))
+    return {"layer_us": sec * 1e6, "launches_per_layer": 2 + 2 * T,
+            "decode_tokens_per_s": B * T / sec, "prefill_flops": flops, "decode_kv_bytes": kv}
 
 
 # ----------------------------------------------------------------------------- CPU oracle legs
@@ -403,6 +438,8 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--headline-only", action="store_true",
                     help="skip the secondary workloads and the CPU baseline")
+    ap.add_argument("--only", choices=("prefill", "gpt2", "paged", "int8"),
+                    help="run one secondary workload alone (for profiling) and print its result")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -429,6 +466,20 @@ def main():
         dist.init_process_group("nccl", device_id=device)
     peaks, peak_src = load_peaks()
     w = wl.MISTRAL_GQA_DECODE
+    if args.only:
+        res = {"only": args.only}
+        if args.only == "prefill":
+            res.update(measure_prefill(wl.MHA7B_PREFILL, args.steps, device, torch))
+        elif args.only == "gpt2":
+            res.update(measure_gpt2_layer(wl.GPT2_LAYER, args.steps, device, torch))
+        else:
+            ow = wl.PAGED_LONG_DECODE if args.only == "paged" else wl.INT8_DECODE
+            orig = DecodeRig(ow, device, copies=1)
+            sd = measure_decode(orig, args.steps, args.warmup, with_append=False)
+            res.update(decode_kernel_us=sd * 1e6, kv_bytes=orig.kv_bytes,
+                       frac=(orig.kv_bytes + orig.io_bytes) / sd / 1e9 / peaks["hbm_gbs"])
+        print(json.dumps(res), flush=True)
+        return
 
     rig = DecodeRig(w, device)
     if dist:
@@ -491,6 +542,8 @@ def main():
             pf.update(frac=pf["tflops"] / peaks["bf16_tflops"], peak=peaks["bf16_tflops"],
                       peak_source=peak_src, bound="tensor")
         extra[pw.name] = dict(pw.as_config(), **pf)
+        gw = wl.GPT2_LAYER
+        extra[gw.name] = dict(gw.as_config(), **measure_gpt2_layer(gw, 50, device, torch))
         # paged long-context decode
         pl = wl.PAGED_LONG_DECODE
         prig = DecodeRig(pl, device, copies=1)

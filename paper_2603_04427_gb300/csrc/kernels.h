@@ -68,6 +68,7 @@ struct PrefillParams {
   int causal;
   float scale_log2;
   int num_sms;
+  int head_group;  // (b, h) pairs per L2 group, set by the launcher
 };
 
 cudaError_t launch_prefill(const PrefillParams& p, cudaStream_t stream, int* unsupported);

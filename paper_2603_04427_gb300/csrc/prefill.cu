@@ -28,6 +28,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "common.cuh"
@@ -120,6 +121,42 @@ __device__ __forceinline__ void tmem_ld64(uint32_t taddr, uint32_t* v) {
       : "r"(taddr), "r"(taddr + 32)
       : "memory");
 }
+// 128 consecutive 32-bit columns (four loads, one wait).
+__device__ __forceinline__ void tmem_ld128(uint32_t taddr, uint32_t* v) {
+  tmem_ld64(taddr, v);
+  tmem_ld64(taddr + 64, v + 64);
+}
+
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;"
+      : "=l"(d)
+      : "l"(*reinterpret_cast<uint64_t*>(&a)), "l"(*reinterpret_cast<uint64_t*>(&b)));
+  return *reinterpret_cast<float2*>(&d);
+}
+
+// Maximum of 128 floats held in registers (three-input max tree, few temporaries).
+__device__ __forceinline__ float max128(const uint32_t* v) {
+#define TK_F(i) __uint_as_float(v[i])
+  float a[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i)
+    a[i] = max3f(max3f(TK_F(8 * i), TK_F(8 * i + 1), TK_F(8 * i + 2)),
+                 max3f(TK_F(8 * i + 3), TK_F(8 * i + 4), TK_F(8 * i + 5)),
+                 fmaxf(TK_F(8 * i + 6), TK_F(8 * i + 7)));
+#undef TK_F
+  const float b0 = max3f(a[0], a[1], a[2]), b1 = max3f(a[3], a[4], a[5]);
+  const float b2 = max3f(a[6], a[7], a[8]), b3 = max3f(a[9], a[10], a[11]);
+  const float b4 = max3f(a[12], a[13], a[14]);
+  return fmaxf(max3f(b0, b1, b2), max3f(b3, b4, a[15]));
+}
+
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* v) {
   asm volatile(
       "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
@@ -212,8 +249,13 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int n_qt = (p.S + kBM - 1) / kBM;
   const int BH = p.B * p.Hq;
-  const int qt = n_qt - 1 - static_cast<int>(blockIdx.x / BH);  // heaviest tiles first
-  const int bh = static_cast<int>(blockIdx.x % BH);
+  // CTA order: heads in groups of p.head_group whose K/V stay in L2 together;
+  // inside a group the heaviest (latest) query tiles first.
+  const int grp = static_cast<int>(blockIdx.x / (p.head_group * n_qt));
+  const int rem = static_cast<int>(blockIdx.x - static_cast<long>(grp) * p.head_group * n_qt);
+  const int gsize = min(p.head_group, BH - grp * p.head_group);
+  const int qt = n_qt - 1 - rem / gsize;
+  const int bh = grp * p.head_group + rem % gsize;
   const int b = bh / p.Hq, h = bh % p.Hq;
   const int kv_plane = b * p.Hkv + h / (p.Hq / p.Hkv);
   const int n_kv_all = (p.S + kBN - 1) / kBN;
@@ -311,19 +353,15 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       const int kv0 = j * kBN;
       const bool masked = (p.causal && kv0 + kBN - 1 > qt * kBM) || (kv0 + kBN > p.S);
       const int lim = min(p.S - kv0, p.causal ? row - kv0 + 1 : kBN);  // visible columns
-      // pass 1: tile max of the raw scores
-      float mx = -INFINITY;
+      // the whole S row of this thread: 128 fp32 scores
+      uint32_t v[128];
+      tmem_ld128(tS + lane_off, v);
+      if (masked) {
 #pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        uint32_t v[64];
-        tmem_ld64(tS + lane_off + 64 * c, v);
-#pragma unroll
-        for (int i = 0; i < 64; ++i) {
-          const float s = __uint_as_float(v[i]);
-          if (!masked || 64 * c + i < lim) mx = fmaxf(mx, s);
-        }
+        for (int i = 0; i < 128; ++i)
+          if (i >= lim) v[i] = 0xff800000u;  // -inf: masked keys get weight exp2(-inf) = 0
       }
-      const float mt = mx * sl2;
+      const float mt = max128(v) * sl2;  // tile max in log2 units (scale > 0)
       const bool resc = mt > m_used + kRescaleThreshold;
       float alpha = 1.f;
       if (resc) {
@@ -331,42 +369,39 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
         m_used = mt;
       }
       l *= alpha;
-      if (j > 0 && __any_sync(0xffffffffu, resc)) {
-        // O *= alpha; the previous P V product is complete (the S_j commit covers it)
-#pragma unroll
-        for (int c = 0; c < DV / 32; ++c) {
-          uint32_t v[32];
-          tmem_ld32(tO + lane_off + 32 * c, v);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
-          tmem_st32(tO + lane_off + 32 * c, v);
-        }
-      }
-      // pass 2: P = exp2(s * scale log2e - m) as bf16 pairs into TMEM columns [0, 64)
-      const float neg_m = -m_used;
-      float lsum0 = 0.f, lsum1 = 0.f;
+      // P = exp2(s * scale log2e - m) as bf16 pairs into TMEM columns [0, 64)
+      const float2 sl2x2 = make_float2(sl2, sl2), negm2 = make_float2(-m_used, -m_used);
+      float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                       make_float2(0.f, 0.f)};
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
         uint32_t pk[32];
-        uint32_t v[64];
-        tmem_ld64(tS + lane_off + 64 * c, v);
 #pragma unroll
-        for (int i = 0; i < 64; i += 2) {
-          const int col = 64 * c + i;
-          float p0 = fast_exp2(fmaf(__uint_as_float(v[i]), sl2, neg_m));
-          float p1 = fast_exp2(fmaf(__uint_as_float(v[i + 1]), sl2, neg_m));
-          if (masked) {
-            if (col >= lim) p0 = 0.f;
-            if (col + 1 >= lim) p1 = 0.f;
-          }
-          lsum0 += p0;
-          lsum1 += p1;
-          __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);  // low half = column col
-          pk[i / 2] = *reinterpret_cast<uint32_t*>(&pr);
+        for (int i = 0; i < 32; ++i) {
+          const int e = 64 * c + 2 * i;
+          const float2 t = ffma2(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])),
+                                 sl2x2, negm2);
+          const float2 pr = make_float2(fast_exp2(t.x), fast_exp2(t.y));
+          acc[i & 3] = fadd2(acc[i & 3], pr);
+          __nv_bfloat162 b2 = __floats2bfloat162_rn(pr.x, pr.y);  // low half = column e
+          pk[i] = *reinterpret_cast<uint32_t*>(&b2);
         }
         tmem_st32(tS + lane_off + 32 * c, pk);
       }
-      l += lsum0 + lsum1;
+      const float2 s01 = fadd2(acc[0], acc[1]), s23 = fadd2(acc[2], acc[3]);
+      if (j > 0 && __any_sync(0xffffffffu, resc)) {
+        // O *= alpha (after P, so the scores no longer occupy registers); the previous
+        // P V product is complete (the S_j commit covers it)
+#pragma unroll
+        for (int c = 0; c < DV / 32; ++c) {
+          uint32_t o[32];
+          tmem_ld32(tO + lane_off + 32 * c, o);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+          tmem_st32(tO + lane_off + 32 * c, o);
+        }
+      }
+      l += (s01.x + s01.y) + (s23.x + s23.y);
       tmem_wait_st();
       tc_fence_before();
       mbar_arrive(p_full);
@@ -467,8 +502,12 @@ cudaError_t launch_t(const PrefillParams& p, cudaStream_t stream) {
   if (e != cudaSuccess) return e;
   const long n_qt = (p.S + kBM - 1) / kBM;
   const long grid = n_qt * p.B * p.Hq;
+  PrefillParams pp = p;
+  // about 48 MB of K/V per head group
+  const long head_bytes = static_cast<long>(p.S) * (R + DV) * 2;
+  pp.head_group = static_cast<int>(std::max(1L, std::min<long>(p.B * p.Hq, (48L << 20) / head_bytes)));
   if (grid > 0x7fffffffL) return cudaErrorInvalidConfiguration;
-  kern<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(maps, p);
+  kern<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(maps, pp);
   return cudaGetLastError();
 }
 

@@ -14,7 +14,7 @@ import numpy as np
 import pytest
 import torch
 
-from _helpers import f64, parity, require_gpu, round_bf16
+from _helpers import f64, parity, parity_bf16, require_gpu
 from oracle import attention as oa
 from paper_2603_04427_gb300 import binding as tb
 from paper_2603_04427_gb300 import inputs
@@ -54,7 +54,7 @@ def test_prefill_lengths_and_bf16_output(S):
     q, k, v = _qkv(B, hq, hkv, S, r, dv, seed=S)
     out = _prefill(q, k, v, dtype=torch.bfloat16)
     ref = oa.attention_prefill(f64(q), f64(k), f64(v), 1 / math.sqrt(r))
-    parity(f64(out), round_bf16(ref), what=f"prefill S={S} bf16 out")
+    parity_bf16(f64(out), ref, what=f"prefill S={S} bf16 out")
     # causal row 0 is v[0] (a single visible key)
     assert torch.equal(out[:, :, 0], v[:, :, 0])
 
@@ -128,5 +128,5 @@ def test_7b_mha_prefill_full_size_sampled():
         ref.append(oa.attention_head(f64(q[b, h, i])[None], f64(k[b, h, :i + 1]),
                                      f64(v[b, h, :i + 1]), 1 / math.sqrt(r))[0])
         got.append(f64(out[b, h, i]))
-    parity(np.stack(got), round_bf16(np.stack(ref)), what="7b prefill sampled")
+    parity_bf16(np.stack(got), np.stack(ref), what="7b prefill sampled")
     assert torch.isfinite(out.float()).all()
