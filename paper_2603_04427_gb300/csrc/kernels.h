@@ -16,8 +16,7 @@ struct DecodeParams {
   const int32_t* seq_lens;   // [B]
   void* out;                 // [B][Hq][DV]
   int out_f32;
-  float* part_o;       // [B][Hkv][n_split][G][DV] unnormalised partial outputs
-  float* part_ml;      // [B][Hkv][n_split][G][2] (running max in log2 units, sum)
+  float* part;         // [n_cta][2][record] partial (o, m, l) of pairs that straddle CTAs
   int32_t* counters;   // [B][Hkv] arrival counters, zero between launches
   int* err;            // device error word
   int B, Hq, Hkv, R, DV, G;
@@ -25,18 +24,17 @@ struct DecodeParams {
   int capacity;        // contiguous
   int page_size, page_shift, num_pages, max_pages;  // paged (page_size 0 = contiguous)
   int max_seq_len;
-  int n_split;         // grid.x
-  int split_chunks;    // 64-token chunks per split
+  int n_cta;           // grid size (one persistent CTA per SM)
   float scale_log2;    // scale * log2(e)
 };
 
-// Split plan shared by tk_decode_workspace_size and tk_attn_decode.
+// Launch plan shared by tk_decode_workspace_size and tk_attn_decode.
 struct DecodePlan {
-  int n_split;
-  int split_chunks;
-  size_t off_counters, off_ml, off_o, bytes;
+  int n_cta;
+  size_t off_counters, off_part, bytes;
 };
-DecodePlan plan_decode(int B, int Hq, int Hkv, int DV, int max_seq_len, int num_sms);
+DecodePlan plan_decode(int B, int Hq, int Hkv, int R, int DV, bool k_int8, int num_sms);
+int decode_max_batch();
 
 cudaError_t launch_decode(const DecodeParams& p, cudaStream_t stream, int* unsupported);
 

@@ -182,8 +182,8 @@ size_t tk_decode_workspace_size(const tk_cache_desc* desc, int32_t max_seq_len) 
   if (check_desc(desc) != TK_OK || max_seq_len < 0) return 0;
   DeviceInfo* dev;
   if (device_info(&dev) != TK_OK) return 0;
-  return tk::plan_decode(desc->batch, desc->h_q, desc->h_kv, desc->d_v, max_seq_len,
-                         dev->num_sms).bytes;
+  return tk::plan_decode(desc->batch, desc->h_q, desc->h_kv, desc->r, desc->d_v,
+                         desc->k_dtype == TK_I8, dev->num_sms).bytes;
 }
 
 tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k_cache,
@@ -204,8 +204,8 @@ tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k
     return fail(TK_ERR_INVALID_ARG, "q / out must be 16-byte aligned");
   DeviceInfo* dev;
   if ((s = device_info(&dev)) != TK_OK) return s;
-  const tk::DecodePlan pl =
-      tk::plan_decode(desc->batch, desc->h_q, desc->h_kv, desc->d_v, max_seq_len, dev->num_sms);
+  const tk::DecodePlan pl = tk::plan_decode(desc->batch, desc->h_q, desc->h_kv, desc->r, desc->d_v,
+                                            desc->k_dtype == TK_I8, dev->num_sms);
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
     return fail(TK_ERR_WORKSPACE, "workspace is NULL or not 256-byte aligned");
   if (workspace_bytes < pl.bytes)
@@ -215,8 +215,7 @@ tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k
   p.q = q; p.k = k_cache; p.v = v_cache; p.k_scale = k_scale; p.page_table = page_table;
   p.seq_lens = seq_lens; p.out = out; p.out_f32 = out_dtype == TK_F32;
   p.counters = reinterpret_cast<int32_t*>(ws + pl.off_counters);
-  p.part_ml = reinterpret_cast<float*>(ws + pl.off_ml);
-  p.part_o = reinterpret_cast<float*>(ws + pl.off_o);
+  p.part = reinterpret_cast<float*>(ws + pl.off_part);
   p.err = dev->err;
   p.B = desc->batch; p.Hq = desc->h_q; p.Hkv = desc->h_kv; p.R = desc->r; p.DV = desc->d_v;
   p.G = desc->h_q / desc->h_kv;
@@ -226,11 +225,12 @@ tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k
   p.page_shift = desc->page_size ? log2i(desc->page_size) : 0;
   p.num_pages = desc->num_pages; p.max_pages = desc->max_pages_per_seq;
   p.max_seq_len = max_seq_len;
-  p.n_split = pl.n_split; p.split_chunks = pl.split_chunks;
+  p.n_cta = pl.n_cta;
   p.scale_log2 = scale * 1.4426950408889634f;
   int uns = 0;
   cudaError_t e = tk::launch_decode(p, static_cast<cudaStream_t>(stream), &uns);
-  if (uns) return fail(TK_ERR_UNSUPPORTED, "decode: no kernel for this shape");
+  if (uns) return fail(TK_ERR_UNSUPPORTED, "decode: no kernel for this shape (batch <= %d)",
+                       tk::decode_max_batch());
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   return TK_OK;
 }

@@ -59,8 +59,9 @@ def test_noalloc_matches_workspace_decode_twice(shape):
 
 def test_noalloc_rejects_shapes_beyond_its_scratch():
     require_gpu()
-    # 1024 sequences x 32 kv heads need about 17 MB of partials, more than the 8 MiB scratch.
-    d = tb.tk_cache_desc(1024, 32, 32, 32, 128, 8192, 0, 0, 0, tb.TK_BF16)
+    # 1024 sequences x 4096 kv heads need 16 MiB of arrival counters alone,
+    # more than the 8 MiB scratch.
+    d = tb.tk_cache_desc(1024, 4096, 4096, 32, 128, 8192, 0, 0, 0, tb.TK_BF16)
     assert tb.tk_decode_workspace_size(d, 8192) > 8 << 20
     fake = torch.empty(16, dtype=torch.uint8, device="cuda")
     L = tb.load_library()
