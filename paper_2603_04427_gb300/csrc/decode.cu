@@ -411,9 +411,11 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
   }
   __syncthreads();
   const long long T = pre[B];
-  // Partition over N = min(grid, T) CTAs so every owning CTA gets at least one
-  // unit and the CTAs sharing a pair are consecutive; the rest own nothing.
-  const int N = static_cast<int>(min(static_cast<long long>(gridDim.x), max(T, 1LL)));
+  // Partition over N = min(grid, ceil(T / 4)) CTAs: every owning CTA gets at
+  // least one unit (four when the cache is small, so short contexts are not
+  // spread over many CTAs) and the CTAs sharing a pair are consecutive; the
+  // rest own nothing.
+  const int N = static_cast<int>(min(static_cast<long long>(gridDim.x), max((T + 3) / 4, 1LL)));
   const long long u_begin = c < N ? T * c / N : T, u_end = c < N ? T * (c + 1) / N : T;
 
   if (warp == kCW) {

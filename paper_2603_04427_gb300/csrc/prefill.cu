@@ -39,9 +39,8 @@ namespace {
 
 constexpr int kBM = 128;          // query rows per tile
 constexpr int kBN = 128;          // keys per kv tile
-constexpr int kStages = 2;
-constexpr int kThreads = 192;     // 4 softmax warps, 1 TMA warp, 1 MMA warp
-constexpr int kTmemCols = 256;
+constexpr int kThreads = 320;     // 2 x 4 softmax warps, 1 TMA warp, 1 MMA warp
+constexpr int kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 // ---------------------------------------------------------------- tcgen05 helpers
@@ -214,12 +213,15 @@ struct PCfg {
   static constexpr int VB = kBN * DV * 2;
   static constexpr int V_NBOX = DV / 64;             // 128-byte-wide boxes of V
   static constexpr int V_BOXB = kBN * 128;
-  static constexpr int OFF_Q = 0;
-  static constexpr int OFF_K = (QB + 1023) / 1024 * 1024;
-  static constexpr int STAGE = (KB + 1023) / 1024 * 1024 + VB;
-  static constexpr int OFF_BAR = OFF_K + kStages * STAGE;
-  static constexpr int SMEM_USED = OFF_BAR + 256;
-  static constexpr int SMEM = SMEM_USED + 1024;      // + slack to align the base to 1 KB
+  static constexpr int QBA = (QB + 1023) / 1024 * 1024;  // one Q tile, 1 KB aligned
+  static constexpr int OFF_Q = 0;                        // two Q tiles
+  static constexpr int OFF_K = 2 * QBA;
+  static constexpr int KBA = (KB + 1023) / 1024 * 1024;
+  static constexpr int STAGE = KBA + VB;
+  static constexpr int NST = (2 * QBA + 3 * STAGE + 2048 <= 200 * 1024) ? 3 : 2;
+  static constexpr int OFF_BAR = OFF_K + NST * STAGE;
+  static constexpr int SMEM = OFF_BAR + 256 + 1024;      // + slack to align the base to 1 KB
+  static_assert(SMEM <= 227 * 1024, "shared memory");
   static constexpr uint32_t IDESC_S = instr_desc(kBM, kBN, false);
   static constexpr uint32_t IDESC_O = instr_desc(kBM, DV, true);
 };
@@ -228,78 +230,93 @@ struct Maps {
   CUtensorMap q, k, v;
 };
 
+// One CTA (one per SM) computes two consecutive 128-row query tiles, A and B,
+// of one (sequence, query head).  They share every K/V tile of the ring, and
+// the MMA warp interleaves them so that one tile's softmax overlaps the other
+// tile's matrix products:
+//   S_A(0) S_B(0) | PV_A(0) S_A(1) PV_B(0) S_B(1) | PV_A(1) S_A(2) PV_B(1) ...
+// TMEM columns: [0,128) S_A (P_A in its first 64 columns), [128,256) S_B,
+// [256,384) O_A, [384,512) O_B.
+//   warps 0-3: softmax and epilogue of tile A (thread i owns row i = TMEM lane i)
+//   warps 4-7: the same for tile B
+//   warp 8: TMA producer (Q tiles once, K/V tiles into an NST-stage ring)
+//   warp 9: MMA issuer
 template <int R, int DV>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, 1)
 prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   using C = PCfg<R, DV>;
+  constexpr int NST = C::NST;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint64_t* q_full = bars + 0;
-  uint64_t* k_full = bars + 1;                  // [kStages]
-  uint64_t* v_full = k_full + kStages;          // [kStages]
-  uint64_t* kv_empty = v_full + kStages;        // [kStages]
-  uint64_t* s_full = kv_empty + kStages;
-  uint64_t* p_full = s_full + 1;
-  uint64_t* o_full = p_full + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_full + 1);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint64_t* k_full = bars + 1;                  // [NST]
+  uint64_t* v_full = k_full + NST;              // [NST]
+  uint64_t* kv_empty = v_full + NST;            // [NST]
+  uint64_t* s_full = kv_empty + NST;            // [2] (tile A, tile B)
+  uint64_t* p_full = s_full + 2;                // [2]
+  uint64_t* o_full = p_full + 2;                // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_full + 2);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int n_qt = (p.S + kBM - 1) / kBM;
+  const int n_tp = (n_qt + 1) / 2;              // query tile pairs
   const int BH = p.B * p.Hq;
   // CTA order: heads in groups of p.head_group whose K/V stay in L2 together;
-  // inside a group the heaviest (latest) query tiles first.
-  const int grp = static_cast<int>(blockIdx.x / (p.head_group * n_qt));
-  const int rem = static_cast<int>(blockIdx.x - static_cast<long>(grp) * p.head_group * n_qt);
+  // inside a group the heaviest (latest) tile pairs first.
+  const int grp = static_cast<int>(blockIdx.x / (p.head_group * n_tp));
+  const int rem = static_cast<int>(blockIdx.x - static_cast<long>(grp) * p.head_group * n_tp);
   const int gsize = min(p.head_group, BH - grp * p.head_group);
-  const int qt = n_qt - 1 - rem / gsize;
+  const int tp = n_tp - 1 - rem / gsize;
   const int bh = grp * p.head_group + rem % gsize;
   const int b = bh / p.Hq, h = bh % p.Hq;
   const int kv_plane = b * p.Hkv + h / (p.Hq / p.Hkv);
+  const int qa = 2 * tp, qb = 2 * tp + 1;
+  const bool has_b = qb < n_qt;
   const int n_kv_all = (p.S + kBN - 1) / kBN;
-  const int n_kv = p.causal ? min(n_kv_all, ((qt + 1) * kBM + kBN - 1) / kBN) : n_kv_all;
+  const int n_a = p.causal ? min(n_kv_all, qa + 1) : n_kv_all;
+  const int n_b = has_b ? (p.causal ? min(n_kv_all, qb + 1) : n_kv_all) : 0;
+  const int n_kv = max(n_a, n_b);
 
   if (tid == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < NST; ++s) {
       mbar_init(&k_full[s], 1);
       mbar_init(&v_full[s], 1);
       mbar_init(&kv_empty[s], 1);
     }
-    mbar_init(s_full, 1);
-    mbar_init(p_full, 128);
-    mbar_init(o_full, 1);
-    *abort_flag = 0;
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(&s_full[x], 1);
+      mbar_init(&p_full[x], 128);
+      mbar_init(&o_full[x], 1);
+    }
     fence_barrier_init();
   }
-  if (warp == 4) {
+  if (warp == 8) {
     tmem_alloc(tmem_slot, kTmemCols);
     tmem_relinquish();
   }
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tS = tmem, tO = tmem + 128;
 
-  if (warp == 4) {
+  if (warp == 8) {
     // ------------------------------------------------------------------ TMA producer
     if (lane == 0) {
       prefetch_map(&maps.q);
       prefetch_map(&maps.k);
       prefetch_map(&maps.v);
-      mbar_arrive_expect_tx(q_full, C::QB);
-      for (int i = 0; i < C::QK_NBOX; ++i)
-        tma_load_3d(smem + C::OFF_Q + i * C::QK_BOXB, &maps.q, i * C::QK_BOX, qt * kBM, bh, q_full);
+      mbar_arrive_expect_tx(q_full, has_b ? 2 * C::QB : C::QB);
+      for (int x = 0; x < (has_b ? 2 : 1); ++x)
+        for (int i = 0; i < C::QK_NBOX; ++i)
+          tma_load_3d(smem + C::OFF_Q + x * C::QBA + i * C::QK_BOXB, &maps.q, i * C::QK_BOX,
+                      (qa + x) * kBM, bh, q_full);
       for (int j = 0; j < n_kv; ++j) {
-        const int st = j % kStages;
-        if (j >= kStages && !mbar_wait(&kv_empty[st], ((j / kStages) - 1) & 1, p.err)) {
-          *abort_flag = 1;
-          break;
-        }
+        const int st = j % NST;
+        if (j >= NST && !mbar_wait(&kv_empty[st], ((j / NST) - 1) & 1, p.err)) break;
         unsigned char* sk = smem + C::OFF_K + st * C::STAGE;
-        unsigned char* sv = sk + (C::KB + 1023) / 1024 * 1024;
+        unsigned char* sv = sk + C::KBA;
         mbar_arrive_expect_tx(&k_full[st], C::KB);
         for (int i = 0; i < C::QK_NBOX; ++i)
           tma_load_3d(sk + i * C::QK_BOXB, &maps.k, i * C::QK_BOX, j * kBN, kv_plane, &k_full[st]);
@@ -308,46 +325,72 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
           tma_load_3d(sv + i * C::V_BOXB, &maps.v, i * 64, j * kBN, kv_plane, &v_full[st]);
       }
     }
-  } else if (warp == 5) {
+  } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      bool ok = mbar_wait(q_full, 0, p.err);
       const uint32_t q_base = smem_addr(smem + C::OFF_Q);
-      for (int j = 0; ok && j < n_kv; ++j) {
-        const int st = j % kStages;
-        const uint32_t ph = (j / kStages) & 1;
-        const uint32_t k_base = smem_addr(smem + C::OFF_K + st * C::STAGE);
-        const uint32_t v_base = k_base + (C::KB + 1023) / 1024 * 1024;
-        if (!(ok = mbar_wait(&k_full[st], ph, p.err))) break;
-        tc_fence_after();
+      auto k_base = [&](int st) { return smem_addr(smem + C::OFF_K + st * C::STAGE); };
+      auto issue_s = [&](int x, int st) {  // S_x = Q_x K^T
 #pragma unroll
         for (int k = 0; k < R / 16; ++k) {
           const uint32_t off = (k / C::KSTEP_PER_BOX) * C::QK_BOXB + (k % C::KSTEP_PER_BOX) * 32;
-          mma_ss(tS, smem_desc(q_base + off, 16, 8 * C::QK_SW, C::QK_LAYOUT),
-                 smem_desc(k_base + off, 16, 8 * C::QK_SW, C::QK_LAYOUT), C::IDESC_S, k > 0);
+          mma_ss(tmem + x * 128, smem_desc(q_base + x * C::QBA + off, 16, 8 * C::QK_SW, C::QK_LAYOUT),
+                 smem_desc(k_base(st) + off, 16, 8 * C::QK_SW, C::QK_LAYOUT), C::IDESC_S, k > 0);
         }
-        tc_commit(s_full);
-        if (!(ok = mbar_wait(p_full, j & 1, p.err))) break;
-        tc_fence_after();
-        if (!(ok = mbar_wait(&v_full[st], ph, p.err))) break;
+        tc_commit(&s_full[x]);
+      };
+      auto issue_pv = [&](int x, int st, bool first) {  // O_x += P_x V
+        const uint32_t v_base = k_base(st) + C::KBA;
 #pragma unroll
         for (int k = 0; k < kBN / 16; ++k)
-          mma_ts(tO, tS + 8 * k, smem_desc(v_base + k * 16 * 128, C::V_BOXB, 1024, 2u),
-                 C::IDESC_O, (j > 0 || k > 0) ? 1u : 0u);
-        tc_commit(&kv_empty[st]);
+          mma_ts(tmem + 256 + x * 128, tmem + x * 128 + 8 * k,
+                 smem_desc(v_base + k * 16 * 128, C::V_BOXB, 1024, 2u), C::IDESC_O,
+                 (!first || k > 0) ? 1u : 0u);
+      };
+      bool ok = mbar_wait(q_full, 0, p.err) && mbar_wait(&k_full[0], 0, p.err);
+      if (ok) {
+        tc_fence_after();
+        issue_s(0, 0);
+        if (has_b) issue_s(1, 0);
       }
-      if (ok) tc_commit(o_full);
-      else *abort_flag = 1;
+      for (int j = 0; ok && j < n_kv; ++j) {
+        const int st = j % NST;
+        const uint32_t ph = (j / NST) & 1;
+        const int stn = (j + 1) % NST;
+        const uint32_t phn = ((j + 1) / NST) & 1;
+        bool v_ready = false;
+        for (int x = 0; x < 2 && ok; ++x) {
+          const int nx = x == 0 ? n_a : n_b;
+          if (j >= nx) continue;
+          if (!(ok = mbar_wait(&p_full[x], j & 1, p.err))) break;
+          if (!v_ready && !(ok = mbar_wait(&v_full[st], ph, p.err))) break;
+          v_ready = true;
+          tc_fence_after();
+          issue_pv(x, st, j == 0);
+          if (j + 1 == nx) {
+            tc_commit(&o_full[x]);
+          } else {
+            if (!(ok = mbar_wait(&k_full[stn], phn, p.err))) break;
+            tc_fence_after();
+            issue_s(x, stn);
+          }
+        }
+        if (ok) tc_commit(&kv_empty[st]);
+      }
     }
   } else {
     // ------------------------------------------------------------------ softmax warps
-    const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
-    const int row = qt * kBM + tid;            // query position of this thread
+    const int x = warp >> 2;                   // 0: tile A, 1: tile B
+    const int nx = x == 0 ? n_a : n_b;
+    const int qt = x == 0 ? qa : qb;
+    const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
+    const uint32_t tS = tmem + x * 128, tO = tmem + 256 + x * 128;
+    const int row = qt * kBM + (tid & 127);    // query position of this thread
     const float sl2 = p.scale_log2;
     float m_used = -INFINITY, l = 0.f;
-    bool ok = true;
-    for (int j = 0; j < n_kv; ++j) {
-      ok = mbar_wait(s_full, j & 1, p.err);
+    bool ok = nx > 0;
+    for (int j = 0; j < nx; ++j) {
+      ok = mbar_wait(&s_full[x], j & 1, p.err);
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after();
       const int kv0 = j * kBN;
@@ -369,7 +412,7 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
         m_used = mt;
       }
       l *= alpha;
-      // P = exp2(s * scale log2e - m) as bf16 pairs into TMEM columns [0, 64)
+      // P = exp2(s * scale log2e - m) as bf16 pairs into TMEM columns [0, 64) of S
       const float2 sl2x2 = make_float2(sl2, sl2), negm2 = make_float2(-m_used, -m_used);
       float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                        make_float2(0.f, 0.f)};
@@ -391,7 +434,7 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       const float2 s01 = fadd2(acc[0], acc[1]), s23 = fadd2(acc[2], acc[3]);
       if (j > 0 && __any_sync(0xffffffffu, resc)) {
         // O *= alpha (after P, so the scores no longer occupy registers); the previous
-        // P V product is complete (the S_j commit covers it)
+        // P V product of this tile is complete (the S_j commit covers it)
 #pragma unroll
         for (int c = 0; c < DV / 32; ++c) {
           uint32_t o[32];
@@ -404,10 +447,10 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       l += (s01.x + s01.y) + (s23.x + s23.y);
       tmem_wait_st();
       tc_fence_before();
-      mbar_arrive(p_full);
+      mbar_arrive(&p_full[x]);
     }
     // epilogue: out = O / l
-    if (ok) ok = mbar_wait(o_full, 0, p.err);
+    if (ok) ok = mbar_wait(&o_full[x], 0, p.err);
     if (__all_sync(0xffffffffu, ok)) {
       tc_fence_after();
       const float inv = 1.f / l;
@@ -440,13 +483,11 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
           }
         }
       }
-    } else {
-      *abort_flag = 1;
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 4) {
+  if (warp == 8) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
@@ -495,13 +536,11 @@ cudaError_t launch_t(const PrefillParams& p, cudaStream_t stream) {
       !make_map(&maps.v, p.v, DV, p.S, p.B * p.Hkv, 64, 128))
     return cudaErrorInvalidValue;
   auto kern = prefill_kernel<R, DV>;
-  // More than a third of the SM's shared memory per CTA keeps it at <= 2 CTAs
-  // per SM, so two 256-column TMEM allocations always fit.
-  const int smem = C::SMEM > 80 * 1024 ? C::SMEM : 80 * 1024;
+  const int smem = C::SMEM;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const long n_qt = (p.S + kBM - 1) / kBM;
-  const long grid = n_qt * p.B * p.Hq;
+  const long grid = (n_qt + 1) / 2 * p.B * p.Hq;  // one CTA per query tile pair
   PrefillParams pp = p;
   // about 48 MB of K/V per head group
   const long head_bytes = static_cast<long>(p.S) * (R + DV) * 2;
