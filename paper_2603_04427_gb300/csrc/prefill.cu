@@ -6,25 +6,25 @@
 // d_v-wide V); Appendix E (prefill is compute-bound; thin keys cut the Q K^T
 // work by d_head / r).
 //
-// One CTA computes one 128-row query tile of one (sequence, query head):
-//   warp 4 (one lane): TMA loads of the Q tile (once) and of 128-row K and V
-//     tiles into a 2-stage shared-memory ring ("full" / "empty" mbarriers).
-//   warp 5 (one lane): issues, per kv tile j,
-//       S_j = Q K_j^T            (M=128, N=128, K=r; bf16 in, fp32 in TMEM)
-//       O  += P_j V_j            (M=128, N=d_v, K=128; P_j read from TMEM)
-//     and signals completion with tcgen05.commit onto mbarriers.
-//   warps 0-3 (thread i owns query row i = TMEM lane i): read S_j from
-//     TMEM, apply the causal / length mask, keep the running max m and sum l
-//     (log2 domain), write P_j = exp2(S_j * scale*log2e - m) as bf16 into the
-//     first 64 TMEM columns of S_j, and at the end write O / l.
+// One CTA per SM computes two consecutive 128-row query tiles, A and B, of one
+// (sequence, query head); they share every 128-row K / V tile of a TMA ring.
+//   warp 8 (one lane): TMA loads of both Q tiles (once) and of the K / V tiles.
+//   warp 9 (whole warp, one elected lane issues): per kv tile j, for x in A, B
+//       O_x += P_x(j) V_j        (M=128, N=d_v, K=128; P_x(j) read from TMEM)
+//       S_x(j+1) = Q_x K_{j+1}^T (M=128, N=128, K=r; bf16 in, fp32 in TMEM)
+//     signalling completion with tcgen05.commit onto mbarriers, so one tile's
+//     softmax overlaps the other tile's matrix products.
+//   warps 0-3 / 4-7 (thread i owns query row i = TMEM lane i of tile A / B):
+//     read S from TMEM, apply the causal / length mask, keep the running max m
+//     and sum l (log2 domain), write P = exp2(S * scale*log2e - m) as bf16 into
+//     the first 64 TMEM columns of S, and at the end write O / l.
 // The running max is updated lazily: O and l are rescaled only when a tile's
 // maximum exceeds the max in use by more than 8 (a factor 256), so the
 // weights stay <= 256 and the result is unchanged (O / l uses one consistent
-// max).  Two CTAs share an SM (256 TMEM columns each), so one CTA's softmax
-// overlaps the other's matrix products.
+// max).
 //
-// TMEM columns per CTA: [0, 128) S (fp32; its first 64 columns hold P as
-// packed bf16 pairs), [128, 128 + d_v) O (fp32).
+// TMEM columns: [0,128) S_A, [128,256) S_B (each: fp32 scores, the first 64
+// columns later hold P as packed bf16 pairs), [256,384) O_A, [384,512) O_B.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -85,6 +85,35 @@ __device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a, uint64_t b, uint3
       "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
       "r"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Variants for the MMA warp, which runs its issue loop with all 32 lanes
+// (warp-uniform control flow and operands): elect.sync picks the one lane
+// that issues the tcgen05 instruction.
+__device__ __forceinline__ void mma_ss_e(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p, e;\n\t.reg .b32 l;\n\telect.sync l|e, 0xffffffff;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "@e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void mma_ts_e(uint32_t d, uint32_t a, uint64_t b, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p, e;\n\t.reg .b32 l;\n\telect.sync l|e, 0xffffffff;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
+      "r"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void tc_commit_e(uint64_t* bar) {
+  asm volatile(
+      "{\n\t.reg .pred e;\n\t.reg .b32 l;\n\telect.sync l|e, 0xffffffff;\n\t"
+      "@e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}" ::"r"(
+          smem_addr(bar))
       : "memory");
 }
 
@@ -190,6 +219,20 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint
          (static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16) |
          (static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46) |
          (static_cast<uint64_t>(layout & 7u) << 61);
+}
+
+// A descriptor as its two 32-bit words.  Advancing the start address by a
+// multiple of 16 bytes is one add to the low word (the 14-bit address field
+// cannot carry: shared-memory addresses stay below 256 KB).
+struct Desc {
+  uint32_t lo, hi;
+  __device__ __forceinline__ uint64_t at(uint32_t byte_off) const {
+    return (static_cast<uint64_t>(hi) << 32) | (lo + (byte_off >> 4));
+  }
+};
+__device__ __forceinline__ Desc make_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo, uint32_t layout) {
+  const uint64_t d = smem_desc(saddr, lbo, sbo, layout);
+  return Desc{static_cast<uint32_t>(d), static_cast<uint32_t>(d >> 32)};
 }
 
 // Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, A K-major.
@@ -327,27 +370,29 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
     }
   } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      const uint32_t q_base = smem_addr(smem + C::OFF_Q);
-      auto k_base = [&](int st) { return smem_addr(smem + C::OFF_K + st * C::STAGE); };
+    {
+      // descriptors of Q tile A and of the K / V tiles of stage 0; other
+      // stages and K steps are start-address offsets from these
+      const Desc dq = make_desc(smem_addr(smem + C::OFF_Q), 16, 8 * C::QK_SW, C::QK_LAYOUT);
+      const Desc dk = make_desc(smem_addr(smem + C::OFF_K), 16, 8 * C::QK_SW, C::QK_LAYOUT);
+      const Desc dv = make_desc(smem_addr(smem + C::OFF_K + C::KBA), C::V_BOXB, 1024, 2u);
       auto issue_s = [&](int x, int st) {  // S_x = Q_x K^T
+        const uint32_t qo = x * C::QBA, ko = st * C::STAGE;
 #pragma unroll
         for (int k = 0; k < R / 16; ++k) {
           const uint32_t off = (k / C::KSTEP_PER_BOX) * C::QK_BOXB + (k % C::KSTEP_PER_BOX) * 32;
-          mma_ss(tmem + x * 128, smem_desc(q_base + x * C::QBA + off, 16, 8 * C::QK_SW, C::QK_LAYOUT),
-                 smem_desc(k_base(st) + off, 16, 8 * C::QK_SW, C::QK_LAYOUT), C::IDESC_S, k > 0);
+          mma_ss_e(tmem + x * 128, dq.at(qo + off), dk.at(ko + off), C::IDESC_S, k > 0);
         }
-        tc_commit(&s_full[x]);
+        tc_commit_e(&s_full[x]);
       };
       auto issue_pv = [&](int x, int st, bool first) {  // O_x += P_x V
-        const uint32_t v_base = k_base(st) + C::KBA;
+        const uint32_t vo = st * C::STAGE;
+        const uint32_t td = tmem + 256 + x * 128, ta = tmem + x * 128;
 #pragma unroll
         for (int k = 0; k < kBN / 16; ++k)
-          mma_ts(tmem + 256 + x * 128, tmem + x * 128 + 8 * k,
-                 smem_desc(v_base + k * 16 * 128, C::V_BOXB, 1024, 2u), C::IDESC_O,
-                 (!first || k > 0) ? 1u : 0u);
+          mma_ts_e(td, ta + 8 * k, dv.at(vo + k * 16 * 128), C::IDESC_O, (!first || k > 0) ? 1u : 0u);
       };
-      bool ok = mbar_wait(q_full, 0, p.err) && mbar_wait(&k_full[0], 0, p.err);
+      bool ok = __all_sync(0xffffffffu, mbar_wait(q_full, 0, p.err) && mbar_wait(&k_full[0], 0, p.err));
       if (ok) {
         tc_fence_after();
         issue_s(0, 0);
@@ -362,20 +407,20 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
         for (int x = 0; x < 2 && ok; ++x) {
           const int nx = x == 0 ? n_a : n_b;
           if (j >= nx) continue;
-          if (!(ok = mbar_wait(&p_full[x], j & 1, p.err))) break;
-          if (!v_ready && !(ok = mbar_wait(&v_full[st], ph, p.err))) break;
+          if (!(ok = __all_sync(0xffffffffu, mbar_wait(&p_full[x], j & 1, p.err)))) break;
+          if (!v_ready && !(ok = __all_sync(0xffffffffu, mbar_wait(&v_full[st], ph, p.err)))) break;
           v_ready = true;
           tc_fence_after();
           issue_pv(x, st, j == 0);
           if (j + 1 == nx) {
-            tc_commit(&o_full[x]);
+            tc_commit_e(&o_full[x]);
           } else {
-            if (!(ok = mbar_wait(&k_full[stn], phn, p.err))) break;
+            if (!(ok = __all_sync(0xffffffffu, mbar_wait(&k_full[stn], phn, p.err)))) break;
             tc_fence_after();
             issue_s(x, stn);
           }
         }
-        if (ok) tc_commit(&kv_empty[st]);
+        if (ok) tc_commit_e(&kv_empty[st]);
       }
     }
   } else {
