@@ -24,6 +24,8 @@ __global__ void __launch_bounds__(kWarps * 32) append_kernel(const AppendParams 
   const long wg = static_cast<long>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
   const long total = static_cast<long>(p.B) * p.Hkv * p.T;
   if (wg >= total) return;
+  pdl_wait();
+  pdl_trigger();
   const int t = static_cast<int>(wg % p.T);
   const int g = static_cast<int>((wg / p.T) % p.Hkv);
   const int b = static_cast<int>(wg / (static_cast<long>(p.T) * p.Hkv));
@@ -99,8 +101,8 @@ cudaError_t launch_t(const AppendParams& p, cudaStream_t s) {
   const long warps = static_cast<long>(p.B) * p.Hkv * p.T;
   const long blocks = (warps + kWarps - 1) / kWarps;
   if (blocks > 0x7fffffffL) return cudaErrorInvalidConfiguration;
-  append_kernel<R, DV, KI8><<<static_cast<unsigned>(blocks), kWarps * 32, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(append_kernel<R, DV, KI8>, dim3(static_cast<unsigned>(blocks)),
+                    dim3(kWarps * 32), 0, s, p);
 }
 
 template <int R, bool KI8>

@@ -83,6 +83,17 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* e
   }
 }
 
+// ---------------------------------------------------------------- dependent launch
+// Kernels launched by launch_pdl may begin while the previous kernel on the
+// stream is still running.  pdl_wait() blocks until that kernel has completed
+// and its memory operations are visible; it must precede every global-memory
+// access of the kernel.  pdl_trigger() allows the next kernel launched this way
+// to begin launching (it still waits in its own pdl_wait()).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---------------------------------------------------------------- bulk copies
 // 1-D bulk copy global -> shared, completion signalled on `bar` as tx bytes.
 // Both addresses 16-byte aligned, bytes a multiple of 16.

@@ -284,56 +284,48 @@ __device__ void merge_segments(const DecodeParams& p, const float* merge, uint64
       last = __shfl_sync(0xffffffffu, last, 0);
       __syncwarp();
       if (last) {
-        // merge the partials of CTAs c_first..c_last, CB segments per batch of loads
+        // merge the partials of CTAs c_first..c_last: each batch of CB partials
+        // is one round of loads (m, l and o together), folded in with an online
+        // rescale; every partial holds at least one token, so its m is finite
         auto slot = [&](int cc) {
           const long long sc = T * cc / N;
           return p.part + (static_cast<long long>(cc) * 2 + (cp <= sc ? 0 : 1)) * C::REC;
         };
         float Mt = -INFINITY, Lt = 0.f;
-        for (int b0 = c_first; b0 <= c_last; b0 += 8) {
-          float mm[8], ll[8];
+        float out[E];
 #pragma unroll
-          for (int k = 0; k < 8; ++k) {
+        for (int i = 0; i < E; ++i) out[i] = 0.f;
+        for (int b0 = c_first; b0 <= c_last; b0 += CB) {
+          float oo[CB][E], mm[CB], ll[CB];
+#pragma unroll
+          for (int k = 0; k < CB; ++k) {
             mm[k] = -INFINITY;
             ll[k] = 0.f;
             if (b0 + k <= c_last) {
               const float* sl = slot(b0 + k);
               mm[k] = __ldcg(sl + G * DV + hh);
               ll[k] = __ldcg(sl + G * DV + G + hh);
-            }
-          }
-          float Mn = Mt;
-#pragma unroll
-          for (int k = 0; k < 8; ++k) Mn = fmaxf(Mn, mm[k]);
-          float Ln = Lt * fast_exp2(Mt - Mn);
-#pragma unroll
-          for (int k = 0; k < 8; ++k) Ln += ll[k] * fast_exp2(mm[k] - Mn);
-          Mt = Mn;
-          Lt = Ln;
-        }
-        float out[E];
-#pragma unroll
-        for (int i = 0; i < E; ++i) out[i] = 0.f;
-        for (int b0 = c_first; b0 <= c_last; b0 += CB) {
-          float oo[CB][E], ww[CB];
-#pragma unroll
-          for (int k = 0; k < CB; ++k) {
-            ww[k] = 0.f;
-            if (b0 + k <= c_last) {
-              const float* sl = slot(b0 + k);
-              ww[k] = __ldcg(sl + G * DV + hh);
               ld_cg_vec<E>(sl + e0, oo[k]);
             } else {
 #pragma unroll
               for (int i = 0; i < E; ++i) oo[k][i] = 0.f;
             }
           }
+          float Mn = Mt;
+#pragma unroll
+          for (int k = 0; k < CB; ++k) Mn = fmaxf(Mn, mm[k]);
+          const float a = Mt == -INFINITY ? 0.f : fast_exp2(Mt - Mn);
+          Lt *= a;
+#pragma unroll
+          for (int i = 0; i < E; ++i) out[i] *= a;
 #pragma unroll
           for (int k = 0; k < CB; ++k) {
-            const float wk2 = (b0 + k <= c_last) ? fast_exp2(ww[k] - Mt) : 0.f;
+            const float wk2 = (b0 + k <= c_last) ? fast_exp2(mm[k] - Mn) : 0.f;
+            Lt += ll[k] * wk2;
 #pragma unroll
             for (int i = 0; i < E; ++i) out[i] += oo[k][i] * wk2;
           }
+          Mt = Mn;
         }
         const float inv = 1.f / Lt;
 #pragma unroll
@@ -369,6 +361,21 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
   const int c = blockIdx.x;
   const int B = p.B, Hkv = p.Hkv;
 
+  if (tid == 0) {
+    for (int s = 0; s < C::NSTAGE; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], kCW);
+    }
+    for (int b2 = 0; b2 < 2; ++b2) {
+      mbar_init(&deposit[b2], kCW);
+      mbar_init(&mfree[b2], 1);
+    }
+    fence_barrier_init();
+  }
+  // everything above touches only shared memory and parameters
+  pdl_wait();
+  pdl_trigger();
+
   // ---- clamped context lengths and prefix sums of units
   int limit = p.max_seq_len;
   if (p.page_size == 0) limit = min(limit, p.capacity);
@@ -380,17 +387,6 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
       L = L < 0 ? 0 : limit;
     }
     lens[b] = L;
-  }
-  if (tid == 0) {
-    for (int s = 0; s < C::NSTAGE; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], kCW);
-    }
-    for (int b2 = 0; b2 < 2; ++b2) {
-      mbar_init(&deposit[b2], kCW);
-      mbar_init(&mfree[b2], 1);
-    }
-    fence_barrier_init();
   }
   __syncthreads();
   if (warp == 0) {
@@ -764,8 +760,7 @@ cudaError_t launch_t(const DecodeParams& p, cudaStream_t stream) {
   const int smem = C::OFF_PRE + (p.B + 1) * 8 + p.B * 4 + 1024;  // + alignment slack
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  kern<<<p.n_cta, kThreads, smem, stream>>>(maps, p);
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3(p.n_cta), dim3(kThreads), smem, stream, maps, p);
 }
 
 // Calls f.template run<R, DV, G, KI8>() for the compiled shape; sets *uns otherwise.
