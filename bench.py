@@ -540,7 +540,9 @@ def main():
         pf = measure_prefill(pw, 20, device, torch)
         if "tflops" in pf:
             pf.update(frac=pf["tflops"] / peaks["bf16_tflops"], peak=peaks["bf16_tflops"],
-                      peak_source=peak_src, bound="tensor")
+                      peak_source=peak_src, bound="tensor",
+                      traffic=recorded_traffic("prefill", pw.name,
+                                               source_hash("prefill.cu", "common.cuh")))
         extra[pw.name] = dict(pw.as_config(), **pf)
         gw = wl.GPT2_LAYER
         extra[gw.name] = dict(gw.as_config(), **measure_gpt2_layer(gw, 50, device, torch))

@@ -116,7 +116,8 @@ typedef struct tk_cache_desc {
  * amax == 0 stores scale 0 and zero codes.
  * n_new == 0 is a no-op.  Positions beyond the capacity (contiguous) or
  * beyond max_pages_per_seq * page_size (paged) are not written and set the
- * device error word.                                                        */
+ * device error word.  Launched with programmatic dependent launch (see
+ * tk_attn_decode).                                                          */
 tk_status tk_kv_append(const tk_cache_desc* desc, void* k_cache, void* v_cache, float* k_scale,
                        const int32_t* page_table, const int32_t* seq_lens, const void* k_new,
                        const void* v_new, int32_t n_new, void* stream);
@@ -143,10 +144,11 @@ tk_status tk_attn_prefill(const void* q, const void* k, const void* v, void* out
 /* Bytes of decode workspace needed for a cache of this shape when no
  * sequence is longer than max_seq_len, on the current device (the split of
  * the context depends on its SM count).  0 means the arguments are invalid.
- * The workspace must be zero-filled once before its first use; every
- * completed tk_attn_decode call leaves it zero-filled again, so it can be
- * reused by later calls in stream order (never by two calls that may run
- * concurrently).                                                            */
+ * The workspace must be zero-filled once before its first use.  It holds
+ * per-(sequence, kv head) arrival counters, which every completed
+ * tk_attn_decode call leaves at zero again, and split partials, which are
+ * scratch; so it can be reused by later calls in stream order (never by two
+ * calls that may run concurrently).                                         */
 size_t tk_decode_workspace_size(const tk_cache_desc* desc, int32_t max_seq_len);
 
 /* Single-token decode attention over the cache (Section 2.1, Eq. 4 with one
@@ -160,8 +162,13 @@ size_t tk_decode_workspace_size(const tk_cache_desc* desc, int32_t max_seq_len);
  *   scale    : multiplies q.k (for int8 keys, q.(code * k_scale))
  *   workspace: device scratch of tk_decode_workspace_size bytes, aligned to
  *              256 bytes (see tk_decode_workspace_size).
+ * batch <= 1024 (the kernel keeps per-sequence prefix sums in shared
+ * memory); a larger batch returns TK_ERR_UNSUPPORTED.
  * The context is split into fixed token ranges processed in parallel and
- * merged in the same launch; results are deterministic run to run.        */
+ * merged in the same launch; results are deterministic run to run.
+ * The kernel is launched with programmatic dependent launch: its CTAs may
+ * start while the previous kernel on `stream` finishes, but they touch
+ * device memory only after that kernel has completed.                      */
 tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k_cache,
                          const void* v_cache, const float* k_scale, const int32_t* page_table,
                          const int32_t* seq_lens, int32_t max_seq_len, void* out,
