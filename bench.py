@@ -207,9 +207,18 @@ class DecodeRig:
         cache.k.copy_(inputs.normal_bf16(cache.k.shape, seed + 1, device=device))
         cache.v.copy_(inputs.normal_bf16(cache.v.shape, seed + 2, device=device))
 
-    def step(self, i, with_append=True):
+    def step(self, i, mode="fused"):
+        """One decode step on copy i: "fused" = tk_attn_decode_append (one launch),
+        "append" = tk_kv_append + tk_attn_decode, "decode" = tk_attn_decode alone."""
         c = self.copies[i % len(self.copies)]
-        if with_append:
+        if mode == "fused":
+            cache = c["cache"]
+            B, hkv = cache.desc.batch, cache.desc.h_kv
+            self.tb.tk_attn_decode_append(cache, c["q"], c["k1"].view(B, hkv, -1),
+                                          c["v1"].view(B, hkv, -1), c["seq_app"], self.max_len,
+                                          c["out"], c["ws"])
+            return
+        if mode == "append":
             self.tb.tk_kv_append(c["cache"], c["k1"], c["v1"], c["seq_app"])
         self.tb.tk_attn_decode(c["cache"], c["q"], c["seq_dec"], self.max_len, c["out"], c["ws"])
 
@@ -255,9 +264,9 @@ def graph_time(torch, enqueue, steps, warmup, max_graph=256):
     return t0.elapsed_time(t1) / 1e3
 
 
-def measure_decode(rig, steps, warmup, with_append=True):
+def measure_decode(rig, steps, warmup, mode="fused"):
     torch = rig.torch
-    sec = graph_time(torch, lambda i: rig.step(i, with_append), steps, warmup)
+    sec = graph_time(torch, lambda i: rig.step(i, mode), steps, warmup)
     return sec / steps
 
 
@@ -345,17 +354,19 @@ def measure_gpt2_layer(w, iters, device, torch):
     zero = torch.zeros(B, dtype=torch.int32, device=device)
     lens = [torch.full((B,), S + t, dtype=torch.int32, device=device) for t in range(T + 1)]
 
+    kd1 = kd.view(T, B, H, r)
+    vd1 = vd.view(T, B, H, dv)
+
     def layer(_):
         tb.tk_attn_prefill(q, k, v, pre)
         tb.tk_kv_append(cache, k, v, zero)
         for t in range(T):
-            tb.tk_kv_append(cache, kd[t], vd[t], lens[t])
-            tb.tk_attn_decode(cache, qd[t], lens[t + 1], S + T, out[t], ws)
+            tb.tk_attn_decode_append(cache, qd[t], kd1[t], vd1[t], lens[t], S + T, out[t], ws)
 
     sec = graph_time(torch, layer, iters, 3, max_graph=4) / iters
     flops = cm.prefill_flops(B, H, S, r, dv)
     kv = sum(cm.decode_kv_bytes([S + t + 1] * B, H, r, dv) for t in range(T))
-    return {"layer_us": sec * 1e6, "launches_per_layer": 2 + 2 * T,
+    return {"layer_us": sec * 1e6, "launches_per_layer": 2 + T,
             "decode_tokens_per_s": B * T / sec, "prefill_flops": flops, "decode_kv_bytes": kv}
 
 
@@ -475,7 +486,7 @@ def main():
         else:
             ow = wl.PAGED_LONG_DECODE if args.only == "paged" else wl.INT8_DECODE
             orig = DecodeRig(ow, device, copies=1)
-            sd = measure_decode(orig, args.steps, args.warmup, with_append=False)
+            sd = measure_decode(orig, args.steps, args.warmup, mode="decode")
             res.update(decode_kernel_us=sd * 1e6, kv_bytes=orig.kv_bytes,
                        frac=(orig.kv_bytes + orig.io_bytes) / sd / 1e9 / peaks["hbm_gbs"])
         print(json.dumps(res), flush=True)
@@ -487,14 +498,15 @@ def main():
     torch.cuda.synchronize()
     clocks = ClockSampler(local)
     clocks.start()
-    sec_step = measure_decode(rig, args.steps, args.warmup, with_append=True)
-    sec_dec = measure_decode(rig, args.steps, args.warmup, with_append=False)
+    sec_step = measure_decode(rig, args.steps, args.warmup, mode="fused")
+    sec_two = measure_decode(rig, args.steps, args.warmup, mode="append")
+    sec_dec = measure_decode(rig, args.steps, args.warmup, mode="decode")
     torch.cuda.synchronize()
     clk = clocks.stop()
     if dist:
-        t = torch.tensor([sec_step, sec_dec], dtype=torch.float64, device=device)
+        t = torch.tensor([sec_step, sec_dec, sec_two], dtype=torch.float64, device=device)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        sec_step, sec_dec = float(t[0]), float(t[1])
+        sec_step, sec_dec, sec_two = float(t[0]), float(t[1]), float(t[2])
     n = world
     value = n * rig.kv_bytes / sec_step / 1e9
     e2e_dt, h2d, d2h = measure_decode_e2e(rig, min(args.steps, 5000))
@@ -509,11 +521,13 @@ def main():
         "warmup": args.warmup, "ms_per_step": sec_step * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": dict(w.as_config(), storage="bf16 K/V, fp32 accumulate, fp32 out",
-                       step="tk_kv_append(1 token) + tk_attn_decode",
+                       step="tk_attn_decode_append: the new token of every sequence is "
+                            "appended inside the decode launch",
                        l2=f"rotating {len(rig.copies)} cache copies "
                           f"({len(rig.copies) * rig.kv_bytes / 1e6:.0f} MB > 4x L2)",
                        parallelism=f"replicas x{n}" if n > 1 else "single GPU"),
         "tokens_per_s": n * w.batch / sec_step,
+        "two_call_step_us": sec_two * 1e6,
         "kv_bytes_per_step": rig.kv_bytes,
         "hbm_frac_of_measured_peak": value / peaks["hbm_gbs"],
         "roofline": {"kernel": "decode_kernel<32,128,4,bf16>", "bound": "hbm",
@@ -525,9 +539,9 @@ def main():
         "e2e": {"value": n * rig.kv_bytes / e2e_dt / 1e9, "unit": "GB/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_dt * 1e3,
-                "how": "pinned host q/k/v of the new token -> device, append + decode, "
+                "how": "pinned host q/k/v of the new token -> device, fused append + decode, "
                        "output -> pinned host, host synchronisation every step"},
-        "gpu_launches": 2 * args.steps,
+        "gpu_launches": args.steps,
         "clocks": clk,
     }
     del rig
@@ -549,8 +563,8 @@ def main():
         # paged long-context decode
         pl = wl.PAGED_LONG_DECODE
         prig = DecodeRig(pl, device, copies=1)
-        s = measure_decode(prig, 200, 20, with_append=True)
-        sd = measure_decode(prig, 200, 20, with_append=False)
+        s = measure_decode(prig, 200, 20, mode="fused")
+        sd = measure_decode(prig, 200, 20, mode="decode")
         extra[pl.name] = dict(pl.as_config(), seq_lens=prig.lens, kv_bytes=prig.kv_bytes,
                               step_us=s * 1e6, gbs=prig.kv_bytes / s / 1e9,
                               decode_kernel_us=sd * 1e6,
@@ -563,8 +577,8 @@ def main():
         for r in iw.r_sweep:
             for k8 in (True, False):
                 rr = DecodeRig(iw, device, copies=1, k_int8=k8, r=r)
-                s = measure_decode(rr, 50, 5, with_append=True)
-                sd = measure_decode(rr, 50, 5, with_append=False)
+                s = measure_decode(rr, 50, 5, mode="fused")
+                sd = measure_decode(rr, 50, 5, mode="decode")
                 sweep.append({"r": r, "k_dtype": "int8" if k8 else "bf16", "kv_bytes": rr.kv_bytes,
                               "step_us": s * 1e6, "gbs": rr.kv_bytes / s / 1e9,
                               "decode_kernel_us": sd * 1e6,

@@ -175,6 +175,29 @@ tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k
                          int32_t out_dtype, float scale, void* workspace,
                          size_t workspace_bytes, void* stream);
 
+/* One decode step with the append fused in: for every sequence, writes the
+ * new token's thin key and value at position seq_lens[b] exactly as
+ * tk_kv_append with n_new = 1 (Section 2.3: the cache keeps k' = x W_K';
+ * int8 keys quantised the same way, bit for bit), then attends q over the
+ * seq_lens[b] + 1 cached tokens exactly as tk_attn_decode with those
+ * lengths (Section 2.1, Eq. 4) -- one launch instead of two.
+ *   seq_lens : device int32 [batch], tokens cached BEFORE the append (not
+ *              modified; the caller advances it by one afterwards)
+ *   k_new    : device bf16 [batch][h_kv][r]    the new thin keys
+ *   v_new    : device bf16 [batch][h_kv][d_v]  the new values
+ *   max_seq_len: host upper bound of seq_lens[b] + 1
+ *   The other arguments, the workspace and the errors are those of
+ *   tk_attn_decode (k_cache, v_cache and k_scale are written).  A sequence
+ *   whose new position does not fit (seq_lens[b] + 1 beyond max_seq_len,
+ *   the capacity or the page table) gets no write, is attended over its
+ *   clamped length and sets the device error word.  The result equals
+ *   tk_kv_append followed by tk_attn_decode bit for bit.                   */
+tk_status tk_attn_decode_append(const tk_cache_desc* desc, const void* q, void* k_cache,
+                                void* v_cache, float* k_scale, const int32_t* page_table,
+                                const int32_t* seq_lens, const void* k_new, const void* v_new,
+                                int32_t max_seq_len, void* out, int32_t out_dtype, float scale,
+                                void* workspace, size_t workspace_bytes, void* stream);
+
 /* Size of the fixed device scratch array used by tk_attn_decode_noalloc. */
 #define TK_DECODE_NOALLOC_SCRATCH_BYTES (8u << 20)
 

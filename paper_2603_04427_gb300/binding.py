@@ -22,7 +22,7 @@ TK_BF16, TK_F32, TK_I8 = 0, 1, 2
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtk.so")
 
 EXPORTED = ("tk_kv_append", "tk_attn_prefill", "tk_decode_workspace_size", "tk_attn_decode",
-            "tk_attn_decode_noalloc", "tk_get_device_error", "tk_status_string", "tk_last_error",
+            "tk_attn_decode_append", "tk_attn_decode_noalloc", "tk_get_device_error", "tk_status_string", "tk_last_error",
             "tk_abi_version")
 
 
@@ -57,6 +57,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tk_attn_prefill": (i32, [vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, i32, vp]),
         "tk_decode_workspace_size": (sz, [dp, i32]),
         "tk_attn_decode": (i32, [dp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp, sz, vp]),
+        "tk_attn_decode_append": (i32, [dp, vp, vp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp,
+                                        sz, vp]),
         "tk_attn_decode_noalloc": (i32, [dp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp]),
         "tk_get_device_error": (i32, [ctypes.POINTER(i32), vp]),
         "tk_status_string": (ctypes.c_char_p, [i32]),
@@ -203,6 +205,35 @@ def tk_attn_decode(cache: ThinKeyCache, q, seq_lens, max_seq_len: int, out, work
                             int(max_seq_len), _ptr(out),
                             TK_F32 if out.dtype == torch.float32 else TK_BF16, scale,
                             _ptr(workspace), workspace.numel(), _stream(stream)), "tk_attn_decode")
+    return out
+
+
+def tk_attn_decode_append(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_seq_len: int, out,
+                          workspace, scale: float | None = None, stream=None):
+    """Append one token per sequence (k_new [B, H_kv, r], v_new [B, H_kv, d_v] bf16) at
+    seq_lens[b] and decode q [B, H_q, r] over the seq_lens[b] + 1 tokens, in one launch."""
+    d = cache.desc
+    dev = cache.k.device
+    _need(q, torch.bfloat16, "q", dev)
+    _need(k_new, torch.bfloat16, "k_new", dev)
+    _need(v_new, torch.bfloat16, "v_new", dev)
+    _need(seq_lens, torch.int32, "seq_lens", dev)
+    _need(workspace, torch.uint8, "workspace", dev)
+    if out.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("out must be float32 or bfloat16")
+    _need(out, out.dtype, "out", dev)
+    if tuple(q.shape) != (d.batch, d.h_q, d.r) or tuple(out.shape) != (d.batch, d.h_q, d.d_v):
+        raise ValueError(f"q {tuple(q.shape)} / out {tuple(out.shape)} do not match the cache")
+    if tuple(k_new.shape) != (d.batch, d.h_kv, d.r) or tuple(v_new.shape) != (d.batch, d.h_kv, d.d_v):
+        raise ValueError(f"k_new {tuple(k_new.shape)} / v_new {tuple(v_new.shape)} do not match the cache")
+    scale = 1.0 / math.sqrt(d.r) if scale is None else float(scale)
+    L = load_library()
+    _check(L.tk_attn_decode_append(ctypes.byref(d), _ptr(q), _ptr(cache.k), _ptr(cache.v),
+                                   _ptr(cache.k_scale), _ptr(cache.page_table), _ptr(seq_lens),
+                                   _ptr(k_new), _ptr(v_new), int(max_seq_len), _ptr(out),
+                                   TK_F32 if out.dtype == torch.float32 else TK_BF16, scale,
+                                   _ptr(workspace), workspace.numel(), _stream(stream)),
+           "tk_attn_decode_append")
     return out
 
 

@@ -3,15 +3,14 @@
 //
 // Paper: Section 2.3 (the thin keys k' = x W_K' are what the cache keeps) and
 // Section 2.4, Eqs. 8-9 (r + d_v values per token and kv head).  The int8
-// variant is the composition with key quantisation of Section 6; the scheme
-// (symmetric absmax per token and kv head, fp32 scale) is this library's
-// reading: scale = amax / 127, code = clamp(rint(k / scale), -127, 127), both
-// divisions in IEEE binary32 (this file is compiled without fast-math).
+// variant is the composition with key quantisation of Section 6 (the scheme
+// is in kv_row.cuh).
 //
 // One warp per (b, g, t): 16-byte vector loads and stores for bf16 rows; for
 // int8 keys a warp max-reduction gives amax.
 #include "common.cuh"
 #include "kernels.h"
+#include "kv_row.cuh"
 
 namespace tk {
 namespace {
@@ -52,48 +51,9 @@ __global__ void __launch_bounds__(kWarps * 32) append_kernel(const AppendParams 
     row = (static_cast<size_t>(page) * p.Hkv + g) * p.page_size + (pos & (p.page_size - 1));
   }
   const size_t src = (static_cast<size_t>(b) * p.Hkv + g) * p.T + t;
-
-  // Values: d_v bf16 = 2 * DV bytes, 16 bytes per lane.
-  {
-    constexpr int NV = 2 * DV / 16;
-    const uint4* s = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(p.v_new) +
-                                                    src * 2 * DV);
-    uint4* d = reinterpret_cast<uint4*>(static_cast<unsigned char*>(p.v) + row * 2 * DV);
-    if (lane < NV) d[lane] = s[lane];
-  }
-  if constexpr (!KI8) {
-    constexpr int NK = 2 * R / 16;
-    const uint4* s = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(p.k_new) +
-                                                    src * 2 * R);
-    uint4* d = reinterpret_cast<uint4*>(static_cast<unsigned char*>(p.k) + row * 2 * R);
-    if (lane < NK) d[lane] = s[lane];
-  } else {
-    // Each lane holds EPL = ceil(R / 32) consecutive key elements.
-    constexpr int EPL = R >= 32 ? R / 32 : 1;
-    const __nv_bfloat16* s = static_cast<const __nv_bfloat16*>(p.k_new) + src * R;
-    float x[EPL];
-    float amax = 0.f;
-#pragma unroll
-    for (int e = 0; e < EPL; ++e) {
-      const int c = lane * EPL + e;
-      x[e] = c < R ? __bfloat162float(s[c]) : 0.f;
-      amax = fmaxf(amax, fabsf(x[e]));
-    }
-#pragma unroll
-    for (int off = 16; off >= 1; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-    const float scale = amax / 127.0f;  // IEEE binary32 division
-    int8_t* d = static_cast<int8_t*>(p.k) + row * R;
-#pragma unroll
-    for (int e = 0; e < EPL; ++e) {
-      const int c = lane * EPL + e;
-      if (c < R) {
-        float code = 0.f;
-        if (scale != 0.f) code = fminf(fmaxf(rintf(x[e] / scale), -127.f), 127.f);
-        d[c] = static_cast<int8_t>(code);
-      }
-    }
-    if (lane == 0) p.k_scale[row] = scale;
-  }
+  write_kv_row<R, DV, KI8>(p.k, p.v, p.k_scale, row,
+                           static_cast<const unsigned char*>(p.k_new) + src * 2 * R,
+                           static_cast<const unsigned char*>(p.v_new) + src * 2 * DV, lane);
 }
 
 template <int R, int DV, bool KI8>

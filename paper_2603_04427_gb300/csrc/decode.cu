@@ -41,6 +41,7 @@
 
 #include "common.cuh"
 #include "kernels.h"
+#include "kv_row.cuh"
 
 namespace tk {
 namespace {
@@ -382,6 +383,7 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
   else limit = min(limit, p.max_pages * p.page_size);
   for (int b = tid; b < B; b += kThreads) {
     int L = p.seq_lens[b];
+    if (p.fuse_append && L >= 0) ++L;  // the appended token is part of the context
     if (L < 0 || L > limit) {
       record_error(p.err, TK_DEVERR_INDEX);
       L = L < 0 ? 0 : limit;
@@ -424,6 +426,45 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
     if (lane == 0) {
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.k)) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.v)) : "memory");
+    }
+    if (p.fuse_append && u_begin < u_end) {
+      // Append fused into the decode: the CTA that reads the last chunk of a
+      // (b, g) pair first writes that pair's new token at position
+      // seq_lens[b] (exactly as the append kernel does), then orders the
+      // writes before its own TMA reads of the chunk with a proxy fence.  No
+      // other CTA reads that chunk.
+      Walker wk;
+      wk.seek(u_begin, pre, lens, B, Hkv);
+      while (true) {
+        const long long last = wk.cp + wk.nb - 1;
+        if (last >= u_end) break;  // this pair's last chunk belongs to a later CTA
+        const int pos = wk.Lb - 1;
+        if (p.seq_lens[wk.b] == pos) {  // not clamped: the new token fits
+          long long row = -1;
+          if (ps == 0) {
+            row = (static_cast<long long>(wk.b) * Hkv + wk.g) * p.capacity + pos;
+          } else {
+            const int page = p.page_table[static_cast<long long>(wk.b) * p.max_pages + (pos >> p.page_shift)];
+            if (page >= 0 && page < p.num_pages)
+              row = (static_cast<long long>(page) * Hkv + wk.g) * ps + (pos & (ps - 1));
+            else if (lane == 0)
+              record_error(p.err, TK_DEVERR_INDEX);
+          }
+          if (row >= 0) {
+            const long long src = static_cast<long long>(wk.b) * Hkv + wk.g;
+            write_kv_row<R, DV, KI8>(const_cast<void*>(p.k), const_cast<void*>(p.v),
+                                     const_cast<float*>(p.k_scale), static_cast<size_t>(row),
+                                     static_cast<const unsigned char*>(p.k_new) + src * 2 * R,
+                                     static_cast<const unsigned char*>(p.v_new) + src * 2 * DV, lane);
+          }
+        }
+        if (last + 1 >= u_end) break;
+        wk.chunk = wk.nb - 1;
+        wk.next(pre, lens, Hkv);
+      }
+      asm volatile("fence.proxy.async.global;" ::: "memory");
+      __syncwarp();
+      asm volatile("fence.proxy.async.global;" ::: "memory");
     }
     bool ok = true;
     for (long long w0 = u_begin; ok && w0 < u_end; w0 += 32) {

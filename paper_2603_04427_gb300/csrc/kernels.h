@@ -45,6 +45,12 @@ struct DecodeParams {
   int max_seq_len;
   int n_cta;           // grid size (one persistent CTA per SM)
   float scale_log2;    // scale * log2(e)
+  // append fused into the decode: seq_lens are the lengths before the append,
+  // the new token of (b, g) (k_new [B][Hkv][R], v_new [B][Hkv][DV]) is
+  // written at position seq_lens[b] and attended to with the cached ones
+  int fuse_append;
+  const void* k_new;
+  const void* v_new;
 };
 
 // Launch plan shared by tk_decode_workspace_size and tk_attn_decode.

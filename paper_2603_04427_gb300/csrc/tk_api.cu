@@ -186,11 +186,13 @@ size_t tk_decode_workspace_size(const tk_cache_desc* desc, int32_t max_seq_len) 
                          desc->k_dtype == TK_I8, dev->num_sms).bytes;
 }
 
-tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k_cache,
-                         const void* v_cache, const float* k_scale, const int32_t* page_table,
-                         const int32_t* seq_lens, int32_t max_seq_len, void* out,
-                         int32_t out_dtype, float scale, void* workspace,
-                         size_t workspace_bytes, void* stream) {
+namespace {
+tk_status decode_impl(const tk_cache_desc* desc, const void* q, const void* k_cache,
+                      const void* v_cache, const float* k_scale, const int32_t* page_table,
+                      const int32_t* seq_lens, const void* k_new, const void* v_new,
+                      int32_t max_seq_len, void* out, int32_t out_dtype, float scale,
+                      void* workspace, size_t workspace_bytes, void* stream) {
+  const bool fuse = k_new != nullptr || v_new != nullptr;
   tk_status s = check_desc(desc);
   if (s != TK_OK) return s;
   if (max_seq_len < 0) return fail(TK_ERR_INVALID_ARG, "max_seq_len=%d", max_seq_len);
@@ -202,6 +204,9 @@ tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k
   if (!q || !out || !seq_lens) return fail(TK_ERR_INVALID_ARG, "q / out / seq_lens is NULL");
   if (!aligned16(q) || !aligned16(out))
     return fail(TK_ERR_INVALID_ARG, "q / out must be 16-byte aligned");
+  if (fuse && (!k_new || !v_new)) return fail(TK_ERR_INVALID_ARG, "k_new / v_new is NULL");
+  if (fuse && (!aligned16(k_new) || !aligned16(v_new)))
+    return fail(TK_ERR_INVALID_ARG, "k_new / v_new must be 16-byte aligned");
   DeviceInfo* dev;
   if ((s = device_info(&dev)) != TK_OK) return s;
   const tk::DecodePlan pl = tk::plan_decode(desc->batch, desc->h_q, desc->h_kv, desc->r, desc->d_v,
@@ -227,12 +232,35 @@ tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k
   p.max_seq_len = max_seq_len;
   p.n_cta = pl.n_cta;
   p.scale_log2 = scale * 1.4426950408889634f;
+  p.fuse_append = fuse;
+  p.k_new = k_new;
+  p.v_new = v_new;
   int uns = 0;
   cudaError_t e = tk::launch_decode(p, static_cast<cudaStream_t>(stream), &uns);
   if (uns) return fail(TK_ERR_UNSUPPORTED, "decode: no kernel for this shape (batch <= %d)",
                        tk::decode_max_batch());
   if (e != cudaSuccess) return cuda_fail(e, "decode launch");
   return TK_OK;
+}
+}  // namespace
+
+tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k_cache,
+                         const void* v_cache, const float* k_scale, const int32_t* page_table,
+                         const int32_t* seq_lens, int32_t max_seq_len, void* out,
+                         int32_t out_dtype, float scale, void* workspace,
+                         size_t workspace_bytes, void* stream) {
+  return decode_impl(desc, q, k_cache, v_cache, k_scale, page_table, seq_lens, nullptr, nullptr,
+                     max_seq_len, out, out_dtype, scale, workspace, workspace_bytes, stream);
+}
+
+tk_status tk_attn_decode_append(const tk_cache_desc* desc, const void* q, void* k_cache,
+                                void* v_cache, float* k_scale, const int32_t* page_table,
+                                const int32_t* seq_lens, const void* k_new, const void* v_new,
+                                int32_t max_seq_len, void* out, int32_t out_dtype, float scale,
+                                void* workspace, size_t workspace_bytes, void* stream) {
+  if (!k_new || !v_new) return fail(TK_ERR_INVALID_ARG, "k_new / v_new is NULL");
+  return decode_impl(desc, q, k_cache, v_cache, k_scale, page_table, seq_lens, k_new, v_new,
+                     max_seq_len, out, out_dtype, scale, workspace, workspace_bytes, stream);
 }
 
 tk_status tk_get_device_error(int32_t* code_out, void* stream) {

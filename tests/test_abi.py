@@ -37,7 +37,7 @@ def test_header_declares_the_boundary():
 def test_every_declared_symbol_is_exported(lib):
     for name in _declared():
         assert hasattr(lib, name), name
-    assert set(_declared()) <= set(tb.EXPORTED) | set(_declared())
+    assert set(_declared()) == set(tb.EXPORTED)
 
 
 def test_abi_version_and_status_strings(lib):
@@ -75,6 +75,9 @@ def test_descriptor_validation(lib, kw, status, msg):
     st = lib.tk_attn_decode(ctypes.byref(d), FAKE, FAKE, FAKE, None, None, FAKE, 16, FAKE,
                             tb.TK_F32, 0.1, FAKE, 1 << 20, None)
     assert st == status
+    st = lib.tk_attn_decode_append(ctypes.byref(d), FAKE, FAKE, FAKE, None, None, FAKE, FAKE,
+                                   FAKE, 16, FAKE, tb.TK_F32, 0.1, FAKE, 1 << 20, None)
+    assert st == status
     assert lib.tk_decode_workspace_size(ctypes.byref(d), 16) == 0
 
 
@@ -103,6 +106,22 @@ def test_pointer_and_option_validation(lib):
                               tb.TK_F32, 0.1, FAKE, 1 << 20, None) == tb.TK_ERR_INVALID_ARG
     assert lib.tk_attn_decode(ctypes.byref(d), FAKE, FAKE, FAKE, None, None, FAKE, 16, FAKE,
                               tb.TK_F32, float("nan"), FAKE, 1 << 20, None) == tb.TK_ERR_INVALID_ARG
+
+
+def test_decode_append_validation(lib):
+    d = _desc()
+    mis = ctypes.c_void_p(0x10008)
+    A = lib.tk_attn_decode_append
+    assert A(ctypes.byref(d), FAKE, FAKE, FAKE, None, None, FAKE, None, FAKE, 16, FAKE,
+             tb.TK_F32, 0.1, FAKE, 1 << 20, None) == tb.TK_ERR_INVALID_ARG
+    assert "k_new" in tb.tk_last_error()
+    assert A(ctypes.byref(d), FAKE, FAKE, FAKE, None, None, FAKE, FAKE, mis, 16, FAKE,
+             tb.TK_F32, 0.1, FAKE, 1 << 20, None) == tb.TK_ERR_INVALID_ARG
+    assert "aligned" in tb.tk_last_error()
+    d8 = _desc(k_dtype=tb.TK_I8)
+    assert A(ctypes.byref(d8), FAKE, FAKE, FAKE, None, None, FAKE, FAKE, FAKE, 16, FAKE,
+             tb.TK_F32, 0.1, FAKE, 1 << 20, None) == tb.TK_ERR_INVALID_ARG
+    assert "k_scale" in tb.tk_last_error()
 
 
 def test_prefill_validation(lib):
