@@ -10,7 +10,8 @@
 // (sequence, query head); they share every 128-row K / V tile of a TMA ring.
 //   warp 8 (one lane): TMA loads of both Q tiles (once) and of the K / V tiles.
 //   warp 9 (whole warp, one elected lane issues): per kv tile j, for x in A, B
-//       O_x += P_x(j) V_j        (M=128, N=d_v, K=128; P_x(j) read from TMEM)
+//       O_x += P_x(j) V_j        (M=128, N=d_v, K=128; P_x(j) read from TMEM,
+//                                 in two 64-key halves as the softmax publishes them)
 //       S_x(j+1) = Q_x K_{j+1}^T (M=128, N=128, K=r; bf16 in, fp32 in TMEM)
 //     signalling completion with tcgen05.commit onto mbarriers, so one tile's
 //     softmax overlaps the other tile's matrix products.
@@ -42,6 +43,11 @@ constexpr int kBN = 128;          // keys per kv tile
 constexpr int kThreads = 320;     // 2 x 4 softmax warps, 1 TMA warp, 1 MMA warp
 constexpr int kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
+// P of a tile is published in kParts key ranges, so the P V products of one
+// range run while the softmax computes the next (two halves measured best;
+// four add more handoff latency than they hide).
+constexpr int kParts = 2;
+constexpr int kPartPairs = kBN / 2 / kParts;  // packed bf16 pairs (TMEM columns) per part
 
 // ---------------------------------------------------------------- tcgen05 helpers
 __device__ __forceinline__ void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
@@ -135,6 +141,16 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* v) {
       : "r"(taddr)
       : "memory");
 }
+// 16 consecutive 32-bit columns.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t* v) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15}, [%16];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : TK_R8(0), TK_R8(8)
+      : "r"(taddr)
+      : "memory");
+}
 // 64 consecutive 32-bit columns (two loads, one wait).
 __device__ __forceinline__ void tmem_ld64(uint32_t taddr, uint32_t* v) {
   asm volatile(
@@ -192,6 +208,18 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* v) {
       "%28, %29, %30, %31, %32};" ::"r"(taddr),
       TK_W8(0), TK_W8(8), TK_W8(16), TK_W8(24)
       : "memory");
+}
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      TK_W8(0), TK_W8(8)
+      : "memory");
+}
+template <int N>
+__device__ __forceinline__ void tmem_st(uint32_t taddr, const uint32_t* v) {
+  if constexpr (N == 32) tmem_st32(taddr, v);
+  else tmem_st16(taddr, v);
 }
 __device__ __forceinline__ void tmem_wait_st() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
@@ -298,8 +326,8 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   uint64_t* v_full = k_full + NST;              // [NST]
   uint64_t* kv_empty = v_full + NST;            // [NST]
   uint64_t* s_full = kv_empty + NST;            // [2] (tile A, tile B)
-  uint64_t* p_full = s_full + 2;                // [2]
-  uint64_t* o_full = p_full + 2;                // [2]
+  uint64_t* p_full = s_full + 2;                // [tile][part]: P of one key range
+  uint64_t* o_full = p_full + 2 * kParts;       // [2]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_full + 2);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -331,7 +359,7 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
     }
     for (int x = 0; x < 2; ++x) {
       mbar_init(&s_full[x], 1);
-      mbar_init(&p_full[x], 128);
+      for (int h = 0; h < kParts; ++h) mbar_init(&p_full[kParts * x + h], 128);
       mbar_init(&o_full[x], 1);
     }
     fence_barrier_init();
@@ -385,12 +413,14 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
         }
         tc_commit_e(&s_full[x]);
       };
-      auto issue_pv = [&](int x, int st, bool first) {  // O_x += P_x V
+      auto issue_pv = [&](int x, int st, bool first, int part) {  // O_x += P_x V, one part
         const uint32_t vo = st * C::STAGE;
         const uint32_t td = tmem + 256 + x * 128, ta = tmem + x * 128;
 #pragma unroll
-        for (int k = 0; k < kBN / 16; ++k)
+        for (int kk = 0; kk < kBN / 16 / kParts; ++kk) {
+          const int k = part * (kBN / 16 / kParts) + kk;
           mma_ts_e(td, ta + 8 * k, dv.at(vo + k * 16 * 128), C::IDESC_O, (!first || k > 0) ? 1u : 0u);
+        }
       };
       bool ok = __all_sync(0xffffffffu, mbar_wait(q_full, 0, p.err) && mbar_wait(&k_full[0], 0, p.err));
       if (ok) {
@@ -407,11 +437,16 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
         for (int x = 0; x < 2 && ok; ++x) {
           const int nx = x == 0 ? n_a : n_b;
           if (j >= nx) continue;
-          if (!(ok = __all_sync(0xffffffffu, mbar_wait(&p_full[x], j & 1, p.err)))) break;
+          // each part of P_x(j) feeds its MMAs while the softmax warps compute
+          // the next part
           if (!v_ready && !(ok = __all_sync(0xffffffffu, mbar_wait(&v_full[st], ph, p.err)))) break;
           v_ready = true;
-          tc_fence_after();
-          issue_pv(x, st, j == 0);
+          for (int h = 0; ok && h < kParts; ++h) {
+            if (!(ok = __all_sync(0xffffffffu, mbar_wait(&p_full[kParts * x + h], j & 1, p.err)))) break;
+            tc_fence_after();
+            issue_pv(x, st, j == 0, h);
+          }
+          if (!ok) break;
           if (j + 1 == nx) {
             tc_commit_e(&o_full[x]);
           } else {
@@ -457,16 +492,17 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
         m_used = mt;
       }
       l *= alpha;
-      // P = exp2(s * scale log2e - m) as bf16 pairs into TMEM columns [0, 64) of S
+      // P = exp2(s * scale log2e - m) as bf16 pairs into TMEM columns [0, 64) of S,
+      // published in kParts consecutive key ranges
       const float2 sl2x2 = make_float2(sl2, sl2), negm2 = make_float2(-m_used, -m_used);
       float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                        make_float2(0.f, 0.f)};
 #pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        uint32_t pk[32];
+      for (int c = 0; c < kParts; ++c) {
+        uint32_t pk[kPartPairs];
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const int e = 64 * c + 2 * i;
+        for (int i = 0; i < kPartPairs; ++i) {
+          const int e = 2 * kPartPairs * c + 2 * i;
           const float2 t = ffma2(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])),
                                  sl2x2, negm2);
           const float2 pr = make_float2(fast_exp2(t.x), fast_exp2(t.y));
@@ -474,25 +510,25 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
           __nv_bfloat162 b2 = __floats2bfloat162_rn(pr.x, pr.y);  // low half = column e
           pk[i] = *reinterpret_cast<uint32_t*>(&b2);
         }
-        tmem_st32(tS + lane_off + 32 * c, pk);
+        tmem_st<kPartPairs>(tS + lane_off + kPartPairs * c, pk);
+        if (c == 0 && j > 0 && __any_sync(0xffffffffu, resc)) {
+          // O *= alpha before any P V product of this tile accumulates into it; the
+          // previous one is complete (the S_j commit covers it)
+#pragma unroll 1
+          for (int cc = 0; cc < DV / 16; ++cc) {
+            uint32_t o[16];
+            tmem_ld16(tO + lane_off + 16 * cc, o);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+            tmem_st16(tO + lane_off + 16 * cc, o);
+          }
+        }
+        tmem_wait_st();
+        tc_fence_before();
+        mbar_arrive(&p_full[kParts * x + c]);
       }
       const float2 s01 = fadd2(acc[0], acc[1]), s23 = fadd2(acc[2], acc[3]);
-      if (j > 0 && __any_sync(0xffffffffu, resc)) {
-        // O *= alpha (after P, so the scores no longer occupy registers); the previous
-        // P V product of this tile is complete (the S_j commit covers it)
-#pragma unroll
-        for (int c = 0; c < DV / 32; ++c) {
-          uint32_t o[32];
-          tmem_ld32(tO + lane_off + 32 * c, o);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-          tmem_st32(tO + lane_off + 32 * c, o);
-        }
-      }
       l += (s01.x + s01.y) + (s23.x + s23.y);
-      tmem_wait_st();
-      tc_fence_before();
-      mbar_arrive(&p_full[x]);
     }
     // epilogue: out = O / l
     if (ok) ok = mbar_wait(&o_full[x], 0, p.err);
