@@ -187,12 +187,18 @@ class DecodeRig:
                 vn = inputs.normal_bf16((B, hkv, T, dv), seed + 2, device=device)
                 tb.tk_kv_append(cache, kn, vn, torch.zeros(B, dtype=torch.int32, device=device))
                 del kn, vn
-            q = inputs.normal_bf16((B, hq, self.r), seed + 3, device=device)
-            k1 = inputs.normal_bf16((B, hkv, 1, self.r), seed + 4, device=device)
-            v1 = inputs.normal_bf16((B, hkv, 1, dv), seed + 5, device=device)
+            # the step's inputs (query, new key, new value) in one buffer, so the
+            # end-to-end leg moves them with one host-to-device copy
+            nq, nk, nv = B * hq * self.r, B * hkv * self.r, B * hkv * dv
+            io = torch.empty(nq + nk + nv, dtype=torch.bfloat16, device=device)
+            q, k1, v1 = io[:nq].view(B, hq, self.r), io[nq:nq + nk].view(B, hkv, 1, self.r), \
+                io[nq + nk:].view(B, hkv, 1, dv)
+            q.copy_(inputs.normal_bf16((B, hq, self.r), seed + 3, device=device))
+            k1.copy_(inputs.normal_bf16((B, hkv, 1, self.r), seed + 4, device=device))
+            v1.copy_(inputs.normal_bf16((B, hkv, 1, dv), seed + 5, device=device))
             out = torch.empty(B, hq, dv, dtype=torch.float32, device=device)
             ws = tb.decode_workspace(cache.desc, self.max_len, device=device)
-            self.copies.append(dict(cache=cache, q=q, k1=k1, v1=v1, out=out, ws=ws,
+            self.copies.append(dict(cache=cache, io=io, q=q, k1=k1, v1=v1, out=out, ws=ws,
                                     seq_app=seq_app, seq_dec=seq_dec))
         torch.cuda.synchronize()
         if tb.tk_get_device_error() != 0:
@@ -271,33 +277,40 @@ def measure_decode(rig, steps, warmup, mode="fused"):
 
 
 def measure_decode_e2e(rig, steps):
-    """Through host buffers: per step H2D of q and the new token's k, v from pinned
-    memory, append + decode, D2H of the output, host synchronisation."""
+    """Through host buffers and the public API: per step one H2D copy of the
+    step's query, new key and new value (one pinned buffer), the fused append +
+    decode (a call prepared once, as a serving loop with fixed buffers makes
+    it), a D2H copy of the output and a host synchronisation."""
     torch = rig.torch
-    c = rig.copies[0]
-    hq = c["q"].cpu().pin_memory()
-    hk = c["k1"].cpu().pin_memory()
-    hv = c["v1"].cpu().pin_memory()
-    ho = torch.empty(c["out"].shape, dtype=torch.float32).pin_memory()
+    tb = rig.tb
+    hio = [c["io"].cpu().pin_memory() for c in rig.copies]
+    ho = torch.empty(rig.copies[0]["out"].shape, dtype=torch.float32).pin_memory()
     stream = torch.cuda.Stream()
+    calls = []
+    for c in rig.copies:
+        cache = c["cache"]
+        B, hkv = cache.desc.batch, cache.desc.h_kv
+        calls.append(tb.prepare_decode_append(cache, c["q"], c["k1"].view(B, hkv, -1),
+                                              c["v1"].view(B, hkv, -1), c["seq_app"], rig.max_len,
+                                              c["out"], c["ws"], stream=stream))
     n = max(1, steps)
     with torch.cuda.stream(stream):
         for i in range(min(n, 20)):  # warm-up
-            c["q"].copy_(hq, non_blocking=True)
-            rig.step(0)
+            c = rig.copies[i % len(rig.copies)]
+            c["io"].copy_(hio[i % len(hio)], non_blocking=True)
+            calls[i % len(calls)]()
             ho.copy_(c["out"], non_blocking=True)
             stream.synchronize()
         t0 = time.perf_counter()
         for i in range(n):
-            cc = rig.copies[i % len(rig.copies)]
-            cc["q"].copy_(hq, non_blocking=True)
-            cc["k1"].copy_(hk, non_blocking=True)
-            cc["v1"].copy_(hv, non_blocking=True)
-            rig.step(i)
-            ho.copy_(cc["out"], non_blocking=True)
+            k = i % len(rig.copies)
+            c = rig.copies[k]
+            c["io"].copy_(hio[k], non_blocking=True)
+            calls[k]()
+            ho.copy_(c["out"], non_blocking=True)
             stream.synchronize()
         dt = (time.perf_counter() - t0) / n
-    h2d = hq.numel() * 2 + hk.numel() * 2 + hv.numel() * 2
+    h2d = hio[0].numel() * 2
     d2h = ho.numel() * 4
     return dt, h2d, d2h
 
@@ -539,8 +552,9 @@ def main():
         "e2e": {"value": n * rig.kv_bytes / e2e_dt / 1e9, "unit": "GB/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_dt * 1e3,
-                "how": "pinned host q/k/v of the new token -> device, fused append + decode, "
-                       "output -> pinned host, host synchronisation every step"},
+                "how": "one pinned host buffer with the step's q, k, v -> device, fused "
+                       "append + decode through a prepared binding call, output -> pinned "
+                       "host, host synchronisation every step"},
         "gpu_launches": args.steps,
         "clocks": clk,
     }

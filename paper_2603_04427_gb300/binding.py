@@ -237,6 +237,50 @@ def tk_attn_decode_append(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_se
     return out
 
 
+class PreparedCall:
+    """One entry-point call with its arguments checked and marshalled once.
+
+    For serving loops whose buffers stay fixed between steps: calling the
+    object re-issues the same C call (same pointers, same stream) without the
+    per-call Python checks, and raises TkError on a non-OK status."""
+
+    def __init__(self, name: str, args: tuple, keep: tuple):
+        self._fn = getattr(load_library(), name)
+        self._name = name
+        self._args = args
+        self._keep = keep  # the tensors whose pointers are in args stay alive
+
+    def __call__(self):
+        st = self._fn(*self._args)
+        if st != TK_OK:
+            _check(st, self._name)
+
+
+def prepare_decode_append(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_seq_len: int, out,
+                          workspace, scale: float | None = None, stream=None) -> PreparedCall:
+    """tk_attn_decode_append with every argument checked once (see that function)."""
+    d = cache.desc
+    dev = cache.k.device
+    for t, n in ((q, "q"), (k_new, "k_new"), (v_new, "v_new")):
+        _need(t, torch.bfloat16, n, dev)
+    _need(seq_lens, torch.int32, "seq_lens", dev)
+    _need(workspace, torch.uint8, "workspace", dev)
+    if out.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("out must be float32 or bfloat16")
+    _need(out, out.dtype, "out", dev)
+    if tuple(q.shape) != (d.batch, d.h_q, d.r) or tuple(out.shape) != (d.batch, d.h_q, d.d_v):
+        raise ValueError(f"q {tuple(q.shape)} / out {tuple(out.shape)} do not match the cache")
+    if tuple(k_new.shape) != (d.batch, d.h_kv, d.r) or tuple(v_new.shape) != (d.batch, d.h_kv, d.d_v):
+        raise ValueError(f"k_new {tuple(k_new.shape)} / v_new {tuple(v_new.shape)} do not match the cache")
+    scale = 1.0 / math.sqrt(d.r) if scale is None else float(scale)
+    args = (ctypes.byref(d), _ptr(q), _ptr(cache.k), _ptr(cache.v), _ptr(cache.k_scale),
+            _ptr(cache.page_table), _ptr(seq_lens), _ptr(k_new), _ptr(v_new), int(max_seq_len),
+            _ptr(out), TK_F32 if out.dtype == torch.float32 else TK_BF16, ctypes.c_float(scale),
+            _ptr(workspace), ctypes.c_size_t(workspace.numel()), _stream(stream))
+    return PreparedCall("tk_attn_decode_append", args,
+                        (cache, q, k_new, v_new, seq_lens, out, workspace))
+
+
 def tk_attn_prefill(q, k, v, out, scale: float | None = None, causal: bool = True, stream=None):
     """Prefill: q [B, H_q, S, r], k [B, H_kv, S, r], v [B, H_kv, S, d_v] bf16 -> out [B, H_q, S, d_v]."""
     dev = q.device

@@ -170,3 +170,32 @@ def test_fused_position_beyond_capacity_is_flagged():
     assert torch.equal(cache.k[0], before.k[0]) and torch.equal(cache.v[0], before.v[0])
     assert torch.equal(cache.k[1, :, 10], k1[1]) and torch.equal(cache.v[1, :, 10], v1[1])
     assert torch.isfinite(out).all()
+
+
+def test_prepared_call_equals_direct_call():
+    """binding.prepare_decode_append checks once and re-issues the same call."""
+    require_gpu()
+    B, hq, hkv, r, dv = 4, 32, 8, 32, 128
+    lens = [100, 640, 1, 300]
+    cache, _, _ = _make(B, hq, hkv, r, dv, lens, False, 0, seed=51)
+    other = _clone(cache)
+    q = inputs.normal_bf16((B, hq, r), seed=52, device="cuda")
+    k1 = inputs.normal_bf16((B, hkv, r), seed=53, device="cuda")
+    v1 = inputs.normal_bf16((B, hkv, dv), seed=54, device="cuda")
+    sl = torch.tensor(lens, dtype=torch.int32, device="cuda")
+    out_d = torch.empty(B, hq, dv, device="cuda")
+    out_p = torch.empty(B, hq, dv, device="cuda")
+    tb.tk_attn_decode_append(other, q, k1, v1, sl, 641, out_d, tb.decode_workspace(other.desc, 641))
+    call = tb.prepare_decode_append(cache, q, k1, v1, sl, 641, out_p,
+                                    tb.decode_workspace(cache.desc, 641))
+    call()
+    torch.cuda.synchronize()
+    assert tb.tk_get_device_error() == 0
+    assert torch.equal(out_d, out_p)
+    _same_cache(other, cache)
+    call()  # again: the same token rewritten at the same positions, same result
+    torch.cuda.synchronize()
+    assert torch.equal(out_d, out_p)
+    with pytest.raises(ValueError):
+        tb.prepare_decode_append(cache, q[:, :4], k1, v1, sl, 641, out_p,
+                                 tb.decode_workspace(cache.desc, 641))
