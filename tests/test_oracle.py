@@ -21,6 +21,9 @@ from oracle import cache as oc
 RNG = np.random.default_rng(1234)
 
 
+torch.manual_seed(1234)  # the torch draws below are then the same on every run
+
+
 def _rand(*shape, scale=1.0):
     return RNG.standard_normal(shape) * scale
 
@@ -278,7 +281,8 @@ def test_quantiser_zero_row():
 
 def test_int8_attention_uses_dequantised_keys():
     B, hq, hkv, cap, r, dv = 2, 4, 2, 30, 16, 8
-    kf = torch.randn(B, hkv, cap, r).to(torch.bfloat16).float().numpy()
+    g = torch.Generator().manual_seed(40)
+    kf = torch.randn(B, hkv, cap, r, generator=g).to(torch.bfloat16).float().numpy()
     codes, sc = oc.quantize_int8_per_token(kf)
     q, v = _rand(B, hq, r), _rand(B, hkv, cap, dv)
     lens = [30, 13]
@@ -290,22 +294,91 @@ def test_int8_attention_uses_dequantised_keys():
     assert np.abs(got - ref).max() < 0.05
 
 
+# ---------------------------------------------------------------- int4 keys
+
+def test_int4_quantiser_ties_round_to_even():
+    # amax 7 gives scale exactly 1, so codes are rint(k): ties go to the even code.
+    k = np.array([[7.0, 2.5, 3.5, -2.5, 0.5, 1.5, -0.5, -7.0]], dtype=np.float32)
+    codes, sc = oc.quantize_int4_per_token(k)
+    assert sc[0] == np.float32(1.0)
+    assert codes.tolist() == [[7, 2, 4, -2, 0, 2, 0, -7]]
+
+
+def test_int4_quantiser_closed_form_and_bounds():
+    k = torch.randn(64, 8, 32).to(torch.bfloat16).float().numpy()
+    codes, sc = oc.quantize_int4_per_token(k)
+    amax = np.abs(k).max(axis=-1)
+    assert np.array_equal(sc, (amax / np.float32(7)).astype(np.float32))
+    assert np.abs(codes.astype(int)).max() <= 7
+    idx = np.abs(k).argmax(axis=-1)
+    top = np.take_along_axis(codes, idx[..., None], -1)[..., 0]
+    assert np.array_equal(np.abs(top.astype(int)), np.full(top.shape, 7))
+    err = np.abs(k - codes * sc[..., None].astype(np.float64))
+    assert np.all(err <= sc[..., None] * (0.5 + 1e-5))
+    c2, s2 = oc.quantize_int4_per_token(-k)
+    assert np.array_equal(c2, -codes) and np.array_equal(s2, sc)
+    z, zs = oc.quantize_int4_per_token(np.zeros((2, 32), dtype=np.float32))
+    assert np.all(z == 0) and np.all(zs == 0)
+
+
+def test_int4_packing():
+    # element 2j in the low nibble, 2j+1 in the high nibble, two's complement
+    codes = np.array([[1, -1, 7, -7, 0, -8]], dtype=np.int8)
+    packed = oc.pack_int4(codes)
+    assert packed.tolist() == [[0xF1, 0x97, 0x80]]
+    assert np.array_equal(oc.unpack_int4(packed), codes)
+    rnd = np.random.default_rng(3).integers(-8, 8, size=(5, 4, 64)).astype(np.int8)
+    assert np.array_equal(oc.unpack_int4(oc.pack_int4(rnd)), rnd)
+    assert oc.pack_int4(rnd).shape == (5, 4, 32)
+
+
+def test_int4_attention_uses_dequantised_keys():
+    B, hq, hkv, cap, r, dv = 2, 4, 2, 30, 32, 8
+    g = torch.Generator().manual_seed(41)
+    kf = torch.randn(B, hkv, cap, r, generator=g).to(torch.bfloat16).float().numpy()
+    codes, sc = oc.quantize_int4_per_token(kf)
+    q, v = _rand(B, hq, r), _rand(B, hkv, cap, dv)
+    lens = [30, 13]
+    got = oa.attention_decode(q, oc.unpack_int4(oc.pack_int4(codes)), v, lens, 0.25, k_scale=sc)
+    deq = codes.astype(np.float64) * sc[..., None].astype(np.float64)
+    assert np.array_equal(got, oa.attention_decode(q, deq, v, lens, 0.25))
+    # If every score of a row moves by at most D, every softmax weight ratio
+    # moves by at most exp(2D), so sum_j |p'_j - p_j| <= exp(2D) - 1 and the
+    # output moves by at most max|v| times that.
+    ref = oa.attention_decode(q, kf, v, lens, 0.25)
+    G = hq // hkv
+    for b in range(B):
+        n = lens[b]
+        for h in range(hq):
+            dk = deq[b, h // G, :n] - kf[b, h // G, :n]
+            D = 0.25 * np.abs(dk @ q[b, h]).max()
+            bound = np.abs(v[b, h // G, :n]).max() * (np.exp(2 * D) - 1)
+            assert np.abs(got[b, h] - ref[b, h]).max() <= bound + 1e-12
+
+
 def test_append_contiguous_and_paged_agree():
     B, hkv, r, dv, ps, cap = 2, 2, 8, 4, 4, 16
     lens = np.array([3, 9])
     T = 5
     kn = torch.randn(B, hkv, T, r).to(torch.bfloat16).float().numpy()
     vn = torch.randn(B, hkv, T, dv).to(torch.bfloat16).float().numpy()
-    for int8 in (False, True):
-        kc = np.zeros((B, hkv, cap, r), dtype=np.int8 if int8 else np.float64)
+    for bits in (16, 8, 4):
+        int8 = bits < 16
+        kw = r // 2 if bits == 4 else r
+        kdt = np.float64 if bits == 16 else (np.int8 if bits == 8 else np.uint8)
+        kc = np.zeros((B, hkv, cap, kw), dtype=kdt)
         vc = np.zeros((B, hkv, cap, dv))
         ksc = np.zeros((B, hkv, cap), dtype=np.float32) if int8 else None
-        oc.append_contiguous(kc, vc, lens, kn, vn, ksc)
+        oc.append_contiguous(kc, vc, lens, kn, vn, ksc, k_bits=4 if bits == 4 else 8)
         table = np.array([[5, 1, 7, 3], [0, 2, 4, 6]])
-        kp = np.zeros((8, hkv, ps, r), dtype=kc.dtype)
+        kp = np.zeros((8, hkv, ps, kw), dtype=kc.dtype)
         vp = np.zeros((8, hkv, ps, dv))
         ksp = np.zeros((8, hkv, ps), dtype=np.float32) if int8 else None
-        oc.append_paged(kp, vp, table, lens, ps, kn, vn, ksp)
+        oc.append_paged(kp, vp, table, lens, ps, kn, vn, ksp, k_bits=4 if bits == 4 else 8)
+        if bits == 4:
+            codes, sc = oc.quantize_int4_per_token(kn)
+            assert np.array_equal(oc.unpack_int4(kc[1, :, 9:14]), codes[1])
+            assert np.array_equal(ksc[1, :, 9:14], sc[1])
         for b in range(B):
             n = lens[b] + T
             assert np.array_equal(oa.gather_pages(kp, table[b], n, ps)[:, lens[b]:],
