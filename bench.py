@@ -144,7 +144,7 @@ class DecodeRig:
     buffers; steps rotate over the copies.
     """
 
-    def __init__(self, w, device, copies=None, k_int8=None, r=None):
+    def __init__(self, w, device, copies=None, k_fmt=None, r=None):
         import torch
 
         from paper_2603_04427_gb300 import binding as tb
@@ -152,7 +152,10 @@ class DecodeRig:
         self.tb, self.torch = tb, torch
         self.w = w
         self.r = r or w.r
-        self.k_int8 = w.k_int8 if k_int8 is None else k_int8
+        # key storage: "bf16", "int8" or "int4" (two codes per byte)
+        self.k_fmt = ("int8" if w.k_int8 else "bf16") if k_fmt is None else k_fmt
+        self.k_int8 = self.k_fmt == "int8"
+        self.k_int4 = self.k_fmt == "int4"
         B, hq, hkv, dv = w.batch, w.h_q, w.h_kv, w.d_v
         if w.seq_range:
             self.lens = inputs.uniform_lengths(B, w.seq_range[0], w.seq_range[1], seed=w.seed)
@@ -160,9 +163,9 @@ class DecodeRig:
             self.lens = [w.seq] * B
         self.max_len = max(self.lens)
         from paper_2603_04427_gb300 import cost_model as cm
-        kb = 1 if self.k_int8 else 2
-        self.kv_bytes = cm.decode_kv_bytes(self.lens, hkv, self.r, dv, k_bytes=kb,
-                                           k_scale_bytes=4 if self.k_int8 else 0)
+        k_row = {"bf16": 2 * self.r, "int8": self.r, "int4": self.r // 2}[self.k_fmt]
+        self.kv_bytes = cm.decode_kv_bytes(self.lens, hkv, k_row, dv, k_bytes=1,
+                                           k_scale_bytes=0 if self.k_fmt == "bf16" else 4)
         self.io_bytes = cm.decode_io_bytes(B, hq, self.r, dv, out_bytes=4)
         per_copy = self.kv_bytes
         if copies is None:
@@ -176,12 +179,14 @@ class DecodeRig:
                 table, n_pages = inputs.paged_layout(self.lens, w.page_size, seed=seed)
                 cache = tb.ThinKeyCache.allocate(B, hq, hkv, self.r, dv, page_size=w.page_size,
                                                  num_pages=n_pages, page_table=table,
-                                                 k_int8=self.k_int8, device=device)
+                                                 k_int8=self.k_int8, k_int4=self.k_int4,
+                                                 device=device)
                 self._fill_paged(cache, seed, device)
             else:
                 cap = (self.max_len + 15) // 16 * 16
                 cache = tb.ThinKeyCache.allocate(B, hq, hkv, self.r, dv, capacity=cap,
-                                                 k_int8=self.k_int8, device=device)
+                                                 k_int8=self.k_int8, k_int4=self.k_int4,
+                                                 device=device)
                 T = self.max_len
                 kn = inputs.normal_bf16((B, hkv, T, self.r), seed + 1, device=device)
                 vn = inputs.normal_bf16((B, hkv, T, dv), seed + 2, device=device)
@@ -207,9 +212,8 @@ class DecodeRig:
     def _fill_paged(self, cache, seed, device):
         from paper_2603_04427_gb300 import inputs
         torch = self.torch
-        if self.k_int8:
-            # quantise through the append kernel, one 64-token page column at a time
-            raise NotImplementedError("paged int8 rig is not used by the benchmark")
+        if self.k_fmt != "bf16":
+            raise NotImplementedError("paged quantised-key rig is not used by the benchmark")
         cache.k.copy_(inputs.normal_bf16(cache.k.shape, seed + 1, device=device))
         cache.v.copy_(inputs.normal_bf16(cache.v.shape, seed + 2, device=device))
 
@@ -589,11 +593,13 @@ def main():
         iw = wl.INT8_DECODE
         sweep = []
         for r in iw.r_sweep:
-            for k8 in (True, False):
-                rr = DecodeRig(iw, device, copies=1, k_int8=k8, r=r)
+            for kf in ("int4", "int8", "bf16"):
+                if kf == "int4" and r < 32:
+                    continue
+                rr = DecodeRig(iw, device, copies=1, k_fmt=kf, r=r)
                 s = measure_decode(rr, 50, 5, mode="fused")
                 sd = measure_decode(rr, 50, 5, mode="decode")
-                sweep.append({"r": r, "k_dtype": "int8" if k8 else "bf16", "kv_bytes": rr.kv_bytes,
+                sweep.append({"r": r, "k_dtype": kf, "kv_bytes": rr.kv_bytes,
                               "step_us": s * 1e6, "gbs": rr.kv_bytes / s / 1e9,
                               "decode_kernel_us": sd * 1e6,
                               "decode_kernel_frac": (rr.kv_bytes + rr.io_bytes) / sd / 1e9 / peaks["hbm_gbs"]})

@@ -36,11 +36,12 @@
  *
  * Cache layouts (owned by the caller, described by tk_cache_desc):
  *   contiguous (page_size == 0):
- *     k_cache  [batch][h_kv][capacity][r]   bf16, or int8 codes
- *     k_scale  [batch][h_kv][capacity]      fp32 (int8 keys only)
+ *     k_cache  [batch][h_kv][capacity][r]   bf16, or int8 codes, or
+ *              [batch][h_kv][capacity][r/2] bytes of packed int4 codes
+ *     k_scale  [batch][h_kv][capacity]      fp32 (int8 / int4 keys only)
  *     v_cache  [batch][h_kv][capacity][d_v] bf16
  *   paged (page_size > 0): pools shared by all sequences
- *     k_cache  [num_pages][h_kv][page_size][r]
+ *     k_cache  [num_pages][h_kv][page_size][r] (r/2 bytes for int4 keys)
  *     k_scale  [num_pages][h_kv][page_size]
  *     v_cache  [num_pages][h_kv][page_size][d_v]
  *     page_table [batch][max_pages_per_seq] int32: logical token t of
@@ -71,7 +72,10 @@ typedef enum tk_status {
 typedef enum tk_dtype {
   TK_BF16 = 0, /* bfloat16                                  */
   TK_F32 = 1,  /* IEEE binary32                             */
-  TK_I8 = 2    /* int8 key codes (value = code * k_scale)   */
+  TK_I8 = 2,   /* int8 key codes (value = code * k_scale)   */
+  TK_I4 = 3    /* int4 key codes, two per byte (element 2j in bits 0-3,
+                  2j+1 in bits 4-7, 4-bit two's complement;
+                  value = code * k_scale)                   */
 } tk_dtype;
 
 /* Shape of a thin-key / full-value cache.
@@ -85,7 +89,7 @@ typedef enum tk_dtype {
  *                      {16, 32, 64, 128, 256}
  *   num_pages        : paged only: pages in each pool
  *   max_pages_per_seq: paged only: columns of the page table
- *   k_dtype          : TK_BF16 or TK_I8                                      */
+ *   k_dtype          : TK_BF16, TK_I8 or TK_I4 (TK_I4 needs r >= 32)          */
 typedef struct tk_cache_desc {
   int32_t batch;
   int32_t h_q;
@@ -108,12 +112,14 @@ typedef struct tk_cache_desc {
  *              token t of the new block goes to position seq_lens[b] + t.
  *              Not modified: the caller advances it (e.g. += n_new on the
  *              same stream) before the next call.
- *   k_scale  : device fp32 per-token scales (int8 keys only, else NULL).
+ *   k_scale  : device fp32 per-token scales (int8 / int4 keys only, else NULL).
  *   page_table: device int32 [batch][max_pages_per_seq] (paged only, else NULL).
  * int8 keys are quantised per (token, kv head): amax = max|k|,
  * scale = amax / 127 (binary32 division, round to nearest), code =
  * clamp(rint(k / scale), -127, 127) (binary32 division, ties to even);
- * amax == 0 stores scale 0 and zero codes.
+ * amax == 0 stores scale 0 and zero codes.  int4 keys (Section 6's 4-bit
+ * composition) use the same scheme with 7 in place of 127 (codes in
+ * [-7, 7]), stored two per byte as described at TK_I4.
  * n_new == 0 is a no-op.  Positions beyond the capacity (contiguous) or
  * beyond max_pages_per_seq * page_size (paged) are not written and set the
  * device error word.  Launched with programmatic dependent launch (see

@@ -129,7 +129,7 @@ def attention_prefill_rows(q, k, v, scale: float, rows, causal: bool = True) -> 
 
 
 def dequantize_keys(codes, scales) -> np.ndarray:
-    """int8 key codes [..., r] times their per-token fp32 scale [...] (exact in fp64)."""
+    """int8 or int4 key codes [..., r] times their per-token fp32 scale [...] (exact in fp64)."""
     return np.asarray(codes, dtype=np.float64) * np.asarray(scales, dtype=np.float64)[..., None]
 
 

@@ -17,7 +17,7 @@ from dataclasses import dataclass
 import torch
 
 TK_OK, TK_ERR_INVALID_ARG, TK_ERR_UNSUPPORTED, TK_ERR_WORKSPACE, TK_ERR_CUDA, TK_ERR_DEVICE = range(6)
-TK_BF16, TK_F32, TK_I8 = 0, 1, 2
+TK_BF16, TK_F32, TK_I8, TK_I4 = 0, 1, 2, 3
 
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtk.so")
 
@@ -111,9 +111,9 @@ def _need(t, dtype, name, device=None):
 class ThinKeyCache:
     """Caller-owned thin-key / full-value cache tensors plus their descriptor.
 
-    Contiguous: k [B, H_kv, cap, r] (bf16 or int8), k_scale [B, H_kv, cap] fp32,
-    v [B, H_kv, cap, d_v] bf16.  Paged: pools [P, H_kv, page_size, ...] and a
-    page table [B, max_pages] int32.
+    Contiguous: k [B, H_kv, cap, r] (bf16 or int8; uint8 [B, H_kv, cap, r/2] of
+    packed int4 codes), k_scale [B, H_kv, cap] fp32, v [B, H_kv, cap, d_v] bf16.
+    Paged: pools [P, H_kv, page_size, ...] and a page table [B, max_pages] int32.
     """
     desc: tk_cache_desc
     k: torch.Tensor
@@ -123,7 +123,7 @@ class ThinKeyCache:
 
     @staticmethod
     def allocate(batch, h_q, h_kv, r, d_v, capacity=0, page_size=0, num_pages=0,
-                 page_table=None, k_int8=False, device="cuda", fill=0):
+                 page_table=None, k_int8=False, device="cuda", fill=0, k_int4=False):
         if page_size:
             if page_table is None:
                 raise ValueError("a paged cache needs a page table")
@@ -133,13 +133,15 @@ class ThinKeyCache:
         else:
             lead = (batch, h_kv, capacity)
             max_pages = 0
-        kd = torch.int8 if k_int8 else torch.bfloat16
-        k = torch.full(lead + (r,), fill, dtype=kd, device=device)
+        if k_int8 and k_int4:
+            raise ValueError("k_int8 and k_int4 are exclusive")
+        kd = torch.int8 if k_int8 else (torch.uint8 if k_int4 else torch.bfloat16)
+        k = torch.full(lead + (r // 2 if k_int4 else r,), fill, dtype=kd, device=device)
         v = torch.full(lead + (d_v,), fill, dtype=torch.bfloat16, device=device)
-        ks = torch.zeros(lead, dtype=torch.float32, device=device) if k_int8 else None
+        ks = torch.zeros(lead, dtype=torch.float32, device=device) if (k_int8 or k_int4) else None
         desc = tk_cache_desc(batch, h_q, h_kv, r, d_v, 0 if page_size else capacity, page_size,
                              num_pages if page_size else 0, max_pages,
-                             TK_I8 if k_int8 else TK_BF16)
+                             TK_I8 if k_int8 else (TK_I4 if k_int4 else TK_BF16))
         return ThinKeyCache(desc, k, v, ks, page_table)
 
 

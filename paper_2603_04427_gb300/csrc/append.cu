@@ -17,7 +17,7 @@ namespace {
 
 constexpr int kWarps = 4;
 
-template <int R, int DV, bool KI8>
+template <int R, int DV, int KF>
 __global__ void __launch_bounds__(kWarps * 32) append_kernel(const AppendParams p) {
   const int lane = threadIdx.x & 31;
   const long wg = static_cast<long>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
@@ -51,37 +51,39 @@ __global__ void __launch_bounds__(kWarps * 32) append_kernel(const AppendParams 
     row = (static_cast<size_t>(page) * p.Hkv + g) * p.page_size + (pos & (p.page_size - 1));
   }
   const size_t src = (static_cast<size_t>(b) * p.Hkv + g) * p.T + t;
-  write_kv_row<R, DV, KI8>(p.k, p.v, p.k_scale, row,
+  write_kv_row<R, DV, KF>(p.k, p.v, p.k_scale, row,
                            static_cast<const unsigned char*>(p.k_new) + src * 2 * R,
                            static_cast<const unsigned char*>(p.v_new) + src * 2 * DV, lane);
 }
 
-template <int R, int DV, bool KI8>
+template <int R, int DV, int KF>
 cudaError_t launch_t(const AppendParams& p, cudaStream_t s) {
   const long warps = static_cast<long>(p.B) * p.Hkv * p.T;
   const long blocks = (warps + kWarps - 1) / kWarps;
   if (blocks > 0x7fffffffL) return cudaErrorInvalidConfiguration;
-  return launch_pdl(append_kernel<R, DV, KI8>, dim3(static_cast<unsigned>(blocks)),
+  return launch_pdl(append_kernel<R, DV, KF>, dim3(static_cast<unsigned>(blocks)),
                     dim3(kWarps * 32), 0, s, p);
 }
 
-template <int R, bool KI8>
+template <int R, int KF>
 cudaError_t by_dv(const AppendParams& p, cudaStream_t s, int* uns) {
   switch (p.DV) {
-    case 64: return launch_t<R, 64, KI8>(p, s);
-    case 128: return launch_t<R, 128, KI8>(p, s);
+    case 64: return launch_t<R, 64, KF>(p, s);
+    case 128: return launch_t<R, 128, KF>(p, s);
   }
   *uns = 1;
   return cudaSuccess;
 }
 
-template <bool KI8>
+template <int KF>
 cudaError_t by_r(const AppendParams& p, cudaStream_t s, int* uns) {
   switch (p.R) {
-    case 16: return by_dv<16, KI8>(p, s, uns);
-    case 32: return by_dv<32, KI8>(p, s, uns);
-    case 64: return by_dv<64, KI8>(p, s, uns);
-    case 128: return by_dv<128, KI8>(p, s, uns);
+    case 16:
+      if constexpr (KF != 2) return by_dv<16, KF>(p, s, uns);
+      break;  // int4 keys need r >= 32
+    case 32: return by_dv<32, KF>(p, s, uns);
+    case 64: return by_dv<64, KF>(p, s, uns);
+    case 128: return by_dv<128, KF>(p, s, uns);
   }
   *uns = 1;
   return cudaSuccess;
@@ -92,7 +94,13 @@ cudaError_t by_r(const AppendParams& p, cudaStream_t s, int* uns) {
 cudaError_t launch_append(const AppendParams& p, cudaStream_t stream, int* unsupported) {
   *unsupported = 0;
   if (p.T == 0 || p.B == 0) return cudaSuccess;
-  return p.k_int8 ? by_r<true>(p, stream, unsupported) : by_r<false>(p, stream, unsupported);
+  switch (p.k_fmt) {
+    case 0: return by_r<0>(p, stream, unsupported);
+    case 1: return by_r<1>(p, stream, unsupported);
+    case 2: return by_r<2>(p, stream, unsupported);
+  }
+  *unsupported = 1;
+  return cudaSuccess;
 }
 
 }  // namespace tk

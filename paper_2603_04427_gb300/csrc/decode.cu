@@ -14,7 +14,7 @@
 //
 //   warp 4 (producer): walks the CTA's units and loads each chunk into an
 //     NSTAGE-deep shared-memory ring: the 64 K rows and V rows as TMA tiles
-//     with 32/64/128-byte swizzle (conflict-free ldmatrix), the int8 key scales
+//     with 32/64/128-byte swizzle (conflict-free ldmatrix), the key scales
 //     and the pair's G query rows with 1-D bulk copies.  For paged caches its
 //     32 lanes look up the page ids of the next 32 units in parallel.
 //   warps 0-3 (consumers): warp w owns tokens 16w..16w+15 of every chunk.  With
@@ -22,10 +22,12 @@
 //       S^T (16 tokens x 8 heads) = K (16 x r) Q^T          (k = r)
 //       O^T (d_v x 8 heads)      += V^T (d_v x 16) P^T       (k = 16 tokens)
 //     bf16 operands, fp32 accumulation.  P moves from the S^T accumulator
-//     layout to the B-operand layout with movmatrix.  int8 keys are widened to
-//     bf16 in registers (exactly), with the query's r index permuted to match
-//     the byte order ldmatrix delivers; the per-token scale multiplies the fp32
-//     score.  Scores are kept in log2 units; online softmax per head.
+//     layout to the B-operand layout with movmatrix.  int8 and int4 keys
+//     (Section 6's composition with key quantisation; int4 two codes per byte)
+//     are widened to bf16 in registers (exactly), with the query's r index
+//     permuted to match the code order ldmatrix delivers; the per-token scale
+//     multiplies the fp32 score.  Scores are kept in log2 units; online
+//     softmax per head.
 //   warp 5 (merger): a segment is the run of one pair's chunks inside the
 //     CTA's range.  At a segment end each consumer warp deposits (m, l, O) in a
 //     double-buffered shared-memory record and carries on streaming; the merger
@@ -52,16 +54,18 @@ constexpr int kThreads = (kCW + 2) * 32;    // + one producer warp + one merger 
 constexpr int kMaxBatch = 1024;             // prefix arrays live in shared memory
 constexpr int kCtaSmemTarget = 110 * 1024;  // aim for two CTAs per SM
 
-template <int R, int DV, int G, bool KI8>
+// KF: key format, 0 bf16, 1 int8, 2 int4 (two codes per byte, R >= 32).
+template <int R, int DV, int G, int KF>
 struct Cfg {
-  static constexpr int RB = KI8 ? R : 2 * R;           // bytes per cached key row
+  static constexpr bool KQ = KF != 0;                  // quantised keys with fp32 scales
+  static constexpr int RB = KF == 0 ? 2 * R : (KF == 1 ? R : R / 2);  // bytes per key row
   static constexpr int KSW = RB >= 128 ? 128 : RB;     // K tile swizzle span (16 = none)
   static constexpr int KBOX_N = RB / KSW;              // K boxes per chunk
   static constexpr int KBOX = kChunk * KSW;            // bytes per K box
   static constexpr int VBOX_N = DV / 64;               // V boxes (64 bf16 = 128 bytes wide)
   static constexpr int VBOX = kChunk * 128;
   static constexpr int KB = KBOX_N * KBOX, VB = VBOX_N * VBOX;
-  static constexpr int SB = KI8 ? kChunk * 4 : 0;
+  static constexpr int SB = KQ ? kChunk * 4 : 0;
   static constexpr int QB = (G * R * 2 + 15) / 16 * 16;
   static constexpr int OFF_V = (KB + 1023) / 1024 * 1024;
   static constexpr int OFF_S = OFF_V + VB;
@@ -132,6 +136,24 @@ __device__ __forceinline__ void i8x4_to_bf16(uint32_t w, uint32_t& lo, uint32_t&
   const float bias = 8388736.0f;  // 2^23 + 128
   lo = pack_bf16(__uint_as_float(f0) - bias, __uint_as_float(f1) - bias);
   hi = pack_bf16(__uint_as_float(f2) - bias, __uint_as_float(f3) - bias);
+}
+// Eight int4 codes (one 32-bit word, code i in bits 4i..4i+3, 4-bit two's
+// complement) to four bf16 pairs (codes 0,1), (2,3), (4,5), (6,7), exactly:
+// flipping each code's sign bit gives c + 8 in [0, 15], which becomes the low
+// mantissa bits of bf16 128 (128 + c + 8), and 136 is subtracted.
+__device__ __forceinline__ uint32_t bf16x2_minus136(uint32_t x) {
+  uint32_t d;
+  asm("sub.rn.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(x), "r"(0x43084308u));
+  return d;
+}
+__device__ __forceinline__ void i4x8_to_bf16(uint32_t w, uint32_t& p01, uint32_t& p23,
+                                             uint32_t& p45, uint32_t& p67) {
+  const uint32_t x = w ^ 0x88888888u;
+  const uint32_t k = 0x43004300u;  // bf16 128.0 in both halves
+  p01 = bf16x2_minus136(k | (x & 0xFu) | ((x << 12) & 0xF0000u));
+  p23 = bf16x2_minus136(k | ((x >> 8) & 0xFu) | ((x << 4) & 0xF0000u));
+  p45 = bf16x2_minus136(k | ((x >> 16) & 0xFu) | ((x >> 4) & 0xF0000u));
+  p67 = bf16x2_minus136(k | ((x >> 24) & 0xFu) | ((x >> 12) & 0xF0000u));
 }
 // Byte offset of (row, byte) inside a TMA box whose rows are SPAN bytes wide
 // and swizzled over SPAN bytes (16 = no swizzle).  Box bases are 1 KB aligned.
@@ -219,12 +241,13 @@ __device__ __forceinline__ void write_out(const DecodeParams& p, long long o, fl
 // pairs that straddle CTAs and, on the last arrival, merge all their partials.
 // Lane l owns E = G*DV/32 consecutive elements of the [G][DV] output, all in
 // head (l*E)/DV.
-template <int R, int DV, int G, bool KI8>
+template <int R, int DV, int G, int KF>
 __device__ void merge_segments(const DecodeParams& p, const float* merge, uint64_t* deposit,
                                uint64_t* mfree, const long long* pre, const int* lens,
                                long long T, int N, int c, long long u_begin, long long u_end,
                                int lane) {
-  using C = Cfg<R, DV, G, KI8>;
+  using C = Cfg<R, DV, G, KF>;
+  constexpr bool KI8 = KF != 0;  // quantised keys (int8 or int4)
   constexpr int E = G * DV / 32;
   constexpr int CB = E >= 32 ? 2 : (E >= 16 ? 4 : 8);  // segments loaded per batch
   const int e0 = lane * E, hh = e0 / DV;
@@ -343,10 +366,11 @@ struct DecodeMaps {
   CUtensorMap k, v;
 };
 
-template <int R, int DV, int G, bool KI8>
+template <int R, int DV, int G, int KF>
 __global__ void __launch_bounds__(kThreads, 1)
 decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
-  using C = Cfg<R, DV, G, KI8>;
+  using C = Cfg<R, DV, G, KF>;
+  constexpr bool KI8 = KF != 0;  // quantised keys (int8 or int4)
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -452,7 +476,7 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
           }
           if (row >= 0) {
             const long long src = static_cast<long long>(wk.b) * Hkv + wk.g;
-            write_kv_row<R, DV, KI8>(const_cast<void*>(p.k), const_cast<void*>(p.v),
+            write_kv_row<R, DV, KF>(const_cast<void*>(p.k), const_cast<void*>(p.v),
                                      const_cast<float*>(p.k_scale), static_cast<size_t>(row),
                                      static_cast<const unsigned char*>(p.k_new) + src * 2 * R,
                                      static_cast<const unsigned char*>(p.v_new) + src * 2 * DV, lane);
@@ -551,7 +575,7 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
         else reinterpret_cast<__nv_bfloat16*>(p.out)[o] = __float2bfloat16_rn(0.f);
       }
     }
-    merge_segments<R, DV, G, KI8>(p, merge, deposit, mfree, pre, lens, T, N, c, u_begin, u_end, lane);
+    merge_segments<R, DV, G, KF>(p, merge, deposit, mfree, pre, lens, T, N, c, u_begin, u_end, lane);
     return;
   }
 
@@ -581,13 +605,23 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
     const bool seg_last = (u + 1 == u_end) || wk.chunk + 1 == wk.nb;
     if (seg_first) {
       // B fragments of Q^T: b0b1 = q[head gq][k 2tq, 2tq+1], b2b3 = q[gq][k 2tq+8, +9] of each
-      // 16-wide k step.  For int8 keys the k order follows the bytes ldmatrix delivers:
-      // mma k (2t, 2t+1, 8+2t, 9+2t) <-> r (4t, 4t+1, 4t+2, 4t+3) within the step.
+      // 16-wide k step.  For quantised keys the k order follows the codes ldmatrix
+      // delivers: int8, mma k (2t, 2t+1, 8+2t, 9+2t) <-> r (4t .. 4t+3) within the step;
+      // int4, steps 2c and 2c+1 take r 32c + 8t + {0..3} and 32c + 8t + {4..7}.
 #pragma unroll
       for (int ks = 0; ks < C::KSTEPS; ++ks) {
         const int base = ks * 16;
-        const int k0 = KI8 ? base + 4 * tq : base + 2 * tq;
-        const int k2 = KI8 ? base + 4 * tq + 2 : base + 2 * tq + 8;
+        int k0, k2;
+        if constexpr (KF == 2) {
+          k0 = (ks >> 1) * 32 + (ks & 1) * 4 + 8 * tq;
+          k2 = k0 + 2;
+        } else if constexpr (KF == 1) {
+          k0 = base + 4 * tq;
+          k2 = k0 + 2;
+        } else {
+          k0 = base + 2 * tq;
+          k2 = base + 2 * tq + 8;
+        }
         float x0 = 0.f, x1 = 0.f, x2 = 0.f, x3 = 0.f;
         if (gq < G && !dead) {
           x0 = __bfloat162float(sq[gq * R + k0]);
@@ -635,6 +669,37 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
           uint32_t a0, a1, a2, a3;
           ldsm_x4(addr, a0, a1, a2, a3);
           mma16816(s, a0, a1, a2, a3, qf[ks][0], qf[ks][1]);
+        }
+      } else if constexpr (KF == 2) {
+        // int4 keys: a 16-byte chunk of a row holds 32 codes, two k steps; ldmatrix
+        // hands lane (g, t) codes 8t..8t+7 of row g: 8t..8t+3 feed the first step,
+        // 8t+4..8t+7 the second (the query's r order above matches)
+        if constexpr (C::KSTEPS == 2) {
+          uint32_t w0, w1;
+          ldsm_x2(k_s + swz<C::KSW>(krow, 0), w0, w1);
+          uint32_t x01, x23, x45, x67, y01, y23, y45, y67;
+          i4x8_to_bf16(w0, x01, x23, x45, x67);
+          i4x8_to_bf16(w1, y01, y23, y45, y67);
+          mma16816(s, x01, y01, x23, y23, qf[0][0], qf[0][1]);
+          mma16816(s, x45, y45, x67, y67, qf[1][0], qf[1][1]);
+        } else {
+#pragma unroll
+          for (int kp = 0; kp < C::KSTEPS / 4; ++kp) {
+            const int kc = kp * 2 + (mi >> 1);
+            const uint32_t addr = k_s + (kc / (C::KSW / 16)) * C::KBOX +
+                                  swz<C::KSW>(krow, (kc % (C::KSW / 16)) * 16);
+            uint32_t w0, w1, w2, w3;  // (rows 0-7, chunk 2kp), (8-15, 2kp), (0-7, 2kp+1), (8-15, 2kp+1)
+            ldsm_x4(addr, w0, w1, w2, w3);
+            uint32_t x01, x23, x45, x67, y01, y23, y45, y67;
+            i4x8_to_bf16(w0, x01, x23, x45, x67);
+            i4x8_to_bf16(w1, y01, y23, y45, y67);
+            mma16816(s, x01, y01, x23, y23, qf[4 * kp][0], qf[4 * kp][1]);
+            mma16816(s, x45, y45, x67, y67, qf[4 * kp + 1][0], qf[4 * kp + 1][1]);
+            i4x8_to_bf16(w2, x01, x23, x45, x67);
+            i4x8_to_bf16(w3, y01, y23, y45, y67);
+            mma16816(s, x01, y01, x23, y23, qf[4 * kp + 2][0], qf[4 * kp + 2][1]);
+            mma16816(s, x45, y45, x67, y67, qf[4 * kp + 3][0], qf[4 * kp + 3][1]);
+          }
         }
       } else {
         // int8 keys: a 16-byte chunk of a row holds one k step; ldmatrix hands lane
@@ -784,9 +849,10 @@ bool make_map_2d(CUtensorMap* m, const void* base, bool int8, long long width, l
              CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int R, int DV, int G, bool KI8>
+template <int R, int DV, int G, int KF>
 cudaError_t launch_t(const DecodeParams& p, cudaStream_t stream) {
-  using C = Cfg<R, DV, G, KI8>;
+  using C = Cfg<R, DV, G, KF>;
+  constexpr bool KI8 = KF != 0;  // quantised keys (int8 or int4)
   // cache rows: contiguous [B*Hkv*cap], paged [P*Hkv*page_size]
   const long long rows = p.page_size == 0
                              ? static_cast<long long>(p.B) * p.Hkv * p.capacity
@@ -794,20 +860,21 @@ cudaError_t launch_t(const DecodeParams& p, cudaStream_t stream) {
   if (rows >= (1LL << 31)) return cudaErrorInvalidValue;  // TMA row coordinates are 32-bit
   const int box_rows = (p.page_size == 0 || p.page_size >= kChunk) ? kChunk : p.page_size;
   DecodeMaps maps;
-  if (!make_map_2d(&maps.k, p.k, KI8, R, rows, C::KSW / (KI8 ? 1 : 2), box_rows, C::KSW) ||
+  if (!make_map_2d(&maps.k, p.k, KI8, KF == 2 ? R / 2 : R, rows, C::KSW / (KI8 ? 1 : 2), box_rows,
+                   C::KSW) ||
       !make_map_2d(&maps.v, p.v, false, DV, rows, 64, box_rows, 128))
     return cudaErrorInvalidValue;
-  auto kern = decode_kernel<R, DV, G, KI8>;
+  auto kern = decode_kernel<R, DV, G, KF>;
   const int smem = C::OFF_PRE + (p.B + 1) * 8 + p.B * 4 + 1024;  // + alignment slack
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   return launch_pdl(kern, dim3(p.n_cta), dim3(kThreads), smem, stream, maps, p);
 }
 
-// Calls f.template run<R, DV, G, KI8>() for the compiled shape; sets *uns otherwise.
+// Calls f.template run<R, DV, G, KF>() for the compiled shape; sets *uns otherwise.
 template <typename F>
-auto dispatch(int R, int DV, int G, bool ki8, F&& f, int* uns) {
-  using Ret = decltype(f.template run<16, 64, 1, false>());
+auto dispatch(int R, int DV, int G, int kf, F&& f, int* uns) {
+  using Ret = decltype(f.template run<16, 64, 1, 0>());
 #define TK_G(R_, DV_, K_)                                      \
   switch (G) {                                                 \
     case 1: return f.template run<R_, DV_, 1, K_>();           \
@@ -823,15 +890,18 @@ auto dispatch(int R, int DV, int G, bool ki8, F&& f, int* uns) {
   }
 #define TK_R(K_)                     \
   switch (R) {                       \
-    case 16: { TK_DV(16, K_) } break;  \
     case 32: { TK_DV(32, K_) } break;  \
     case 64: { TK_DV(64, K_) } break;  \
     case 128: { TK_DV(128, K_) } break; \
   }
-  if (ki8) {
-    TK_R(true)
-  } else {
-    TK_R(false)
+  if (kf == 0) {
+    if (R == 16) { TK_DV(16, 0) }
+    TK_R(0)
+  } else if (kf == 1) {
+    if (R == 16) { TK_DV(16, 1) }
+    TK_R(1)
+  } else if (kf == 2) {
+    TK_R(2)  // int4 keys need r >= 32
   }
 #undef TK_R
 #undef TK_DV
@@ -841,14 +911,14 @@ auto dispatch(int R, int DV, int G, bool ki8, F&& f, int* uns) {
 }
 
 struct CtasPerSm {
-  template <int R, int DV, int G, bool K>
+  template <int R, int DV, int G, int K>
   int run() { return Cfg<R, DV, G, K>::CTAS_PER_SM; }
 };
 
 struct Launch {
   const DecodeParams* p;
   cudaStream_t s;
-  template <int R, int DV, int G, bool K>
+  template <int R, int DV, int G, int K>
   cudaError_t run() { return launch_t<R, DV, G, K>(*p, s); }
 };
 
@@ -856,10 +926,10 @@ struct Launch {
 
 int decode_max_batch() { return kMaxBatch; }
 
-DecodePlan plan_decode(int B, int Hq, int Hkv, int R, int DV, bool k_int8, int num_sms) {
+DecodePlan plan_decode(int B, int Hq, int Hkv, int R, int DV, int k_fmt, int num_sms) {
   DecodePlan pl{};
   int uns = 0;
-  const int per_sm = dispatch(R, DV, Hq / Hkv, k_int8, CtasPerSm{}, &uns);
+  const int per_sm = dispatch(R, DV, Hq / Hkv, k_fmt, CtasPerSm{}, &uns);
   pl.n_cta = num_sms * (uns ? 1 : per_sm);
   const int G = Hq / Hkv;
   const size_t rec = (static_cast<size_t>(G) * DV + 2 * G + 3) / 4 * 4;
@@ -876,7 +946,7 @@ cudaError_t launch_decode(const DecodeParams& p, cudaStream_t stream, int* unsup
     *unsupported = 1;
     return cudaSuccess;
   }
-  return dispatch(p.R, p.DV, p.G, p.k_int8 != 0, Launch{&p, stream}, unsupported);
+  return dispatch(p.R, p.DV, p.G, p.k_fmt, Launch{&p, stream}, unsupported);
 }
 
 }  // namespace tk

@@ -39,7 +39,7 @@ struct DecodeParams {
   int32_t* counters;   // [B][Hkv] arrival counters, zero between launches
   int* err;            // device error word
   int B, Hq, Hkv, R, DV, G;
-  int k_int8;
+  int k_fmt;           // key format: 0 bf16, 1 int8, 2 int4 (two codes per byte)
   int capacity;        // contiguous
   int page_size, page_shift, num_pages, max_pages;  // paged (page_size 0 = contiguous)
   int max_seq_len;
@@ -58,7 +58,7 @@ struct DecodePlan {
   int n_cta;
   size_t off_counters, off_part, bytes;
 };
-DecodePlan plan_decode(int B, int Hq, int Hkv, int R, int DV, bool k_int8, int num_sms);
+DecodePlan plan_decode(int B, int Hq, int Hkv, int R, int DV, int k_fmt, int num_sms);
 int decode_max_batch();
 
 cudaError_t launch_decode(const DecodeParams& p, cudaStream_t stream, int* unsupported);
@@ -73,7 +73,7 @@ struct AppendParams {
   const void* v_new;         // bf16 [B][Hkv][T][DV]
   int* err;
   int B, Hkv, R, DV, T;
-  int k_int8;
+  int k_fmt;   // 0 bf16, 1 int8, 2 int4
   int capacity;
   int page_size, page_shift, num_pages, max_pages;
 };

@@ -86,8 +86,10 @@ tk_status check_desc(const tk_cache_desc* d) {
     return fail(TK_ERR_UNSUPPORTED, "h_q/h_kv=%d (supported: 1, 2, 4, 8)", d->h_q / d->h_kv);
   if (!supported_r(d->r)) return fail(TK_ERR_UNSUPPORTED, "r=%d (supported: 16, 32, 64, 128)", d->r);
   if (!supported_dv(d->d_v)) return fail(TK_ERR_UNSUPPORTED, "d_v=%d (supported: 64, 128)", d->d_v);
-  if (d->k_dtype != TK_BF16 && d->k_dtype != TK_I8)
-    return fail(TK_ERR_UNSUPPORTED, "k_dtype=%d (supported: TK_BF16, TK_I8)", d->k_dtype);
+  if (d->k_dtype != TK_BF16 && d->k_dtype != TK_I8 && d->k_dtype != TK_I4)
+    return fail(TK_ERR_UNSUPPORTED, "k_dtype=%d (supported: TK_BF16, TK_I8, TK_I4)", d->k_dtype);
+  if (d->k_dtype == TK_I4 && d->r < 32)
+    return fail(TK_ERR_UNSUPPORTED, "r=%d with TK_I4 keys (supported: 32, 64, 128)", d->r);
   if (d->page_size == 0) {
     if (d->capacity <= 0 || d->capacity % 16 != 0)
       return fail(TK_ERR_INVALID_ARG, "capacity=%d must be a positive multiple of 16", d->capacity);
@@ -102,12 +104,16 @@ tk_status check_desc(const tk_cache_desc* d) {
   return TK_OK;
 }
 
+// Key format index used by the kernels: 0 bf16, 1 int8, 2 int4.
+int key_format(int32_t k_dtype) { return k_dtype == TK_I8 ? 1 : (k_dtype == TK_I4 ? 2 : 0); }
+
 tk_status check_cache_ptrs(const tk_cache_desc* d, const void* k, const void* v, const void* ks,
                            const void* pt) {
   if (!k || !v) return fail(TK_ERR_INVALID_ARG, "k_cache / v_cache is NULL");
   if (!aligned16(k) || !aligned16(v) || (ks && !aligned16(ks)))
     return fail(TK_ERR_INVALID_ARG, "cache pointers must be 16-byte aligned");
-  if (d->k_dtype == TK_I8 && !ks) return fail(TK_ERR_INVALID_ARG, "int8 keys need k_scale");
+  if ((d->k_dtype == TK_I8 || d->k_dtype == TK_I4) && !ks)
+    return fail(TK_ERR_INVALID_ARG, "int8 / int4 keys need k_scale");
   if (d->page_size != 0 && !pt) return fail(TK_ERR_INVALID_ARG, "paged cache needs page_table");
   return TK_OK;
 }
@@ -133,7 +139,7 @@ tk_status tk_kv_append(const tk_cache_desc* desc, void* k_cache, void* v_cache, 
   p.k = k_cache; p.v = v_cache; p.k_scale = k_scale; p.page_table = page_table;
   p.seq_lens = seq_lens; p.k_new = k_new; p.v_new = v_new; p.err = dev->err;
   p.B = desc->batch; p.Hkv = desc->h_kv; p.R = desc->r; p.DV = desc->d_v; p.T = n_new;
-  p.k_int8 = desc->k_dtype == TK_I8;
+  p.k_fmt = key_format(desc->k_dtype);
   p.capacity = desc->capacity;
   p.page_size = desc->page_size;
   p.page_shift = desc->page_size ? log2i(desc->page_size) : 0;
@@ -183,7 +189,7 @@ size_t tk_decode_workspace_size(const tk_cache_desc* desc, int32_t max_seq_len) 
   DeviceInfo* dev;
   if (device_info(&dev) != TK_OK) return 0;
   return tk::plan_decode(desc->batch, desc->h_q, desc->h_kv, desc->r, desc->d_v,
-                         desc->k_dtype == TK_I8, dev->num_sms).bytes;
+                         key_format(desc->k_dtype), dev->num_sms).bytes;
 }
 
 namespace {
@@ -210,7 +216,7 @@ tk_status decode_impl(const tk_cache_desc* desc, const void* q, const void* k_ca
   DeviceInfo* dev;
   if ((s = device_info(&dev)) != TK_OK) return s;
   const tk::DecodePlan pl = tk::plan_decode(desc->batch, desc->h_q, desc->h_kv, desc->r, desc->d_v,
-                                            desc->k_dtype == TK_I8, dev->num_sms);
+                                            key_format(desc->k_dtype), dev->num_sms);
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
     return fail(TK_ERR_WORKSPACE, "workspace is NULL or not 256-byte aligned");
   if (workspace_bytes < pl.bytes)
@@ -224,7 +230,7 @@ tk_status decode_impl(const tk_cache_desc* desc, const void* q, const void* k_ca
   p.err = dev->err;
   p.B = desc->batch; p.Hq = desc->h_q; p.Hkv = desc->h_kv; p.R = desc->r; p.DV = desc->d_v;
   p.G = desc->h_q / desc->h_kv;
-  p.k_int8 = desc->k_dtype == TK_I8;
+  p.k_fmt = key_format(desc->k_dtype);
   p.capacity = desc->capacity;
   p.page_size = desc->page_size;
   p.page_shift = desc->page_size ? log2i(desc->page_size) : 0;

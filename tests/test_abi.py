@@ -66,6 +66,7 @@ FAKE = ctypes.c_void_p(0x10000)  # never dereferenced: validation fails first
     (dict(page_size=48, num_pages=4, max_pages_per_seq=2), tb.TK_ERR_UNSUPPORTED, "page_size"),
     (dict(page_size=64, num_pages=0, max_pages_per_seq=2), tb.TK_ERR_INVALID_ARG, "num_pages"),
     (dict(k_dtype=7), tb.TK_ERR_UNSUPPORTED, "k_dtype"),
+    (dict(k_dtype=tb.TK_I4, r=16), tb.TK_ERR_UNSUPPORTED, "TK_I4"),
 ])
 def test_descriptor_validation(lib, kw, status, msg):
     d = _desc(**kw)
