@@ -108,6 +108,28 @@ def attention_prefill(q, k, v, scale: float, causal: bool = True) -> np.ndarray:
     return out
 
 
+def attention_prefill_cached(q, k, v, seq_lens, scale: float, causal: bool = True) -> np.ndarray:
+    """Prefill of a chunk that continues a cached context (Eqs. 1-4 over the grown context).
+
+    q: [B, H_q, S, r] the chunk's queries; k: [B, H_kv, n, r], v: [B, H_kv, n, d_v]
+    the sequence's keys and values, chunk included (n >= seq_lens[b] + S).
+    Query i of sequence b sits at position seq_lens[b] + i and attends to keys
+    0 .. seq_lens[b] + i (causal) or to all seq_lens[b] + S of them.
+    Returns [B, H_q, S, d_v] float64.
+    """
+    q, k, v = (np.asarray(x, dtype=np.float64) for x in (q, k, v))
+    B, h_q, S, _ = q.shape
+    h_kv = k.shape[1]
+    out = np.zeros((B, h_q, S, v.shape[3]), dtype=np.float64)
+    for b in range(B):
+        n = int(seq_lens[b]) + S
+        for h in range(h_q):
+            g = _kv_head(h, h_q, h_kv)
+            out[b, h] = attention_head(q[b, h], k[b, g, :n], v[b, g, :n], scale,
+                                       causal_offset=int(seq_lens[b]) if causal else None)
+    return out
+
+
 def attention_prefill_rows(q, k, v, scale: float, rows, causal: bool = True) -> np.ndarray:
     """Selected output rows of ``attention_prefill``, each computed on its own.
 

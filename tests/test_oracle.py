@@ -245,6 +245,38 @@ def test_decode_matches_torch_sdpa_ragged():
         np.testing.assert_allclose(got[b:b + 1], want, rtol=1e-10, atol=1e-12)
 
 
+# ---------------------------------------------------------------- prefill over a cache
+
+def test_cached_prefill_reduces_to_prefill_and_decode():
+    B, hq, hkv, S, r, dv = 2, 4, 2, 9, 8, 5
+    L0 = [0, 6]
+    n = max(L0) + S
+    q = _rand(B, hq, S, r)
+    k, v = _rand(B, hkv, n, r), _rand(B, hkv, n, dv)
+    got = oa.attention_prefill_cached(q, k, v, L0, 0.3)
+    # no cached tokens: the plain causal prefill of the chunk
+    np.testing.assert_allclose(got[0], oa.attention_prefill(q[:1], k[:1, :, :S], v[:1, :, :S], 0.3)[0],
+                               rtol=1e-13, atol=1e-14)
+    # each row: decode over the L0 + i + 1 keys it may see
+    for i in range(S):
+        want = oa.attention_decode(q[:, :, i], k, v, [l0 + i + 1 for l0 in L0], 0.3)
+        np.testing.assert_allclose(got[:, :, i], want, rtol=1e-13, atol=1e-14)
+    # non-causal: every row sees all L0 + S keys
+    full = oa.attention_prefill_cached(q, k, v, L0, 0.3, causal=False)
+    for i in range(S):
+        want = oa.attention_decode(q[:, :, i], k, v, [l0 + S for l0 in L0], 0.3)
+        np.testing.assert_allclose(full[:, :, i], want, rtol=1e-13, atol=1e-14)
+
+
+def test_cached_prefill_brute_force():
+    q, k, v = _rand(1, 1, 3, 4), _rand(1, 1, 5, 4), _rand(1, 1, 5, 3)
+    got = oa.attention_prefill_cached(q, k, v, [2], 0.5)
+    for i in range(3):
+        want = brute.head([q[0, 0, i].tolist()], k[0, 0, :3 + i].tolist(),
+                          v[0, 0, :3 + i].tolist(), 0.5)[0][0]
+        np.testing.assert_allclose(got[0, 0, i], want, rtol=1e-12, atol=1e-14)
+
+
 # ---------------------------------------------------------------- int8 keys
 
 def test_quantiser_ties_round_to_even():
