@@ -351,6 +351,32 @@ def measure_prefill(w, iters, device, torch):
     return {"ms": sec * 1e3, "tflops": flops / sec / 1e12, "flops_per_launch": flops}
 
 
+def measure_chunked_prefill(w, iters, device, torch):
+    """A prompt chunk of w.seq tokens after w.cached cached ones: tk_attn_prefill_cached
+    (append of the chunk + attention over the cache), bf16 output."""
+    from paper_2603_04427_gb300 import binding as tb
+    from paper_2603_04427_gb300 import cost_model as cm
+    from paper_2603_04427_gb300 import inputs
+    B, hq, hkv, S, r, dv, L0 = w.batch, w.h_q, w.h_kv, w.seq, w.r, w.d_v, w.cached
+    cache = tb.ThinKeyCache.allocate(B, hq, hkv, r, dv, capacity=L0 + S, device=device)
+    zero = torch.zeros(B, dtype=torch.int32, device=device)
+    tb.tk_kv_append(cache, inputs.normal_bf16((B, hkv, L0, r), w.seed + 1, device=device),
+                    inputs.normal_bf16((B, hkv, L0, dv), w.seed + 2, device=device), zero)
+    q = inputs.normal_bf16((B, hq, S, r), w.seed + 3, device=device)
+    kn = inputs.normal_bf16((B, hkv, S, r), w.seed + 4, device=device)
+    vn = inputs.normal_bf16((B, hkv, S, dv), w.seed + 5, device=device)
+    out = torch.empty(B, hq, S, dv, dtype=torch.bfloat16, device=device)
+    sl = torch.full((B,), L0, dtype=torch.int32, device=device)
+
+    def enq(_):  # the same chunk re-appended at the same positions every time
+        tb.tk_attn_prefill_cached(cache, q, kn, vn, sl, L0 + S, out)
+
+    sec = graph_time(torch, enq, iters, 3, max_graph=16) / iters
+    flops = cm.prefill_flops(B, hq, S, r, dv, cached=L0)
+    return {"ms": sec * 1e3, "tflops": flops / sec / 1e12, "flops_per_call": flops,
+            "cached": L0, "launches": 2}
+
+
 def measure_gpt2_layer(w, iters, device, torch):
     """GPT-2-small layer: causal prefill of S tokens (fp32 out), append of the
     prompt's keys/values, then `decode_steps` x (append 1 token + decode)."""
@@ -466,7 +492,7 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--headline-only", action="store_true",
                     help="skip the secondary workloads and the CPU baseline")
-    ap.add_argument("--only", choices=("prefill", "gpt2", "paged", "int8"),
+    ap.add_argument("--only", choices=("prefill", "chunked", "gpt2", "paged", "int8"),
                     help="run one secondary workload alone (for profiling) and print its result")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -498,6 +524,8 @@ def main():
         res = {"only": args.only}
         if args.only == "prefill":
             res.update(measure_prefill(wl.MHA7B_PREFILL, args.steps, device, torch))
+        elif args.only == "chunked":
+            res.update(measure_chunked_prefill(wl.CHUNKED_PREFILL, args.steps, device, torch))
         elif args.only == "gpt2":
             res.update(measure_gpt2_layer(wl.GPT2_LAYER, args.steps, device, torch))
         else:
@@ -576,6 +604,11 @@ def main():
                       traffic=recorded_traffic("prefill", pw.name,
                                                source_hash("prefill.cu", "common.cuh")))
         extra[pw.name] = dict(pw.as_config(), **pf)
+        cw = wl.CHUNKED_PREFILL
+        cp = measure_chunked_prefill(cw, 20, device, torch)
+        cp.update(frac=cp["tflops"] / peaks["bf16_tflops"], peak=peaks["bf16_tflops"],
+                  peak_source=peak_src, bound="tensor")
+        extra[cw.name] = dict(cw.as_config(), **cp)
         gw = wl.GPT2_LAYER
         extra[gw.name] = dict(gw.as_config(), **measure_gpt2_layer(gw, 50, device, torch))
         # paged long-context decode

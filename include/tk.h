@@ -147,6 +147,32 @@ tk_status tk_attn_prefill(const void* q, const void* k, const void* v, void* out
                           int32_t seq, int32_t r, int32_t d_v, float scale, int32_t causal,
                           void* stream);
 
+/* Prefill of a chunk of `seq` new tokens per sequence against the cache
+ * (Section 2.1, Eqs. 1-4, over a context that continues an existing one):
+ * first writes the chunk's thin keys and values at positions
+ * seq_lens[b] .. seq_lens[b] + seq - 1 exactly as tk_kv_append, then
+ * computes, for query i of the chunk (position seq_lens[b] + i),
+ * attention over the cache's tokens 0 .. seq_lens[b] + i (causal, aligned
+ * to the end of the context) or over all seq_lens[b] + seq of them
+ * (causal == 0).
+ *   q        : device bf16 [batch][h_q][seq][r]       the chunk's queries
+ *   k_new    : device bf16 [batch][h_kv][seq][r]      the chunk's thin keys
+ *   v_new    : device bf16 [batch][h_kv][seq][d_v]    the chunk's values
+ *   seq_lens : device int32 [batch], tokens cached before the chunk (not
+ *              modified; the caller advances it by seq afterwards)
+ *   max_seq_len: host bound of seq_lens[b] + seq
+ *   out      : device [batch][h_q][seq][d_v], TK_BF16 or TK_F32
+ * bf16 keys only (TK_ERR_UNSUPPORTED otherwise): the products run on the
+ * tensor cores from bf16 tiles.  Contiguous or paged caches; a sequence whose
+ * chunk does not fit sets the device error word and is computed over a
+ * clamped context.  seq_lens[b] == 0 gives the plain causal prefill of the
+ * chunk.  Two launches (append, then attention) in stream order.           */
+tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void* k_cache,
+                                 void* v_cache, const int32_t* page_table,
+                                 const int32_t* seq_lens, const void* k_new, const void* v_new,
+                                 int32_t seq, int32_t max_seq_len, void* out, int32_t out_dtype,
+                                 float scale, int32_t causal, void* stream);
+
 /* Bytes of decode workspace needed for a cache of this shape when no
  * sequence is longer than max_seq_len, on the current device (the split of
  * the context depends on its SM count).  0 means the arguments are invalid.

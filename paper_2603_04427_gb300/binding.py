@@ -22,7 +22,7 @@ TK_BF16, TK_F32, TK_I8, TK_I4 = 0, 1, 2, 3
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtk.so")
 
 EXPORTED = ("tk_kv_append", "tk_attn_prefill", "tk_decode_workspace_size", "tk_attn_decode",
-            "tk_attn_decode_append", "tk_attn_decode_noalloc", "tk_get_device_error", "tk_status_string", "tk_last_error",
+            "tk_attn_decode_append", "tk_attn_decode_noalloc", "tk_attn_prefill_cached", "tk_get_device_error", "tk_status_string", "tk_last_error",
             "tk_abi_version")
 
 
@@ -56,6 +56,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tk_kv_append": (i32, [dp, vp, vp, vp, vp, vp, vp, vp, i32, vp]),
         "tk_attn_prefill": (i32, [vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, i32, vp]),
         "tk_decode_workspace_size": (sz, [dp, i32]),
+        "tk_attn_prefill_cached": (i32, [dp, vp, vp, vp, vp, vp, vp, vp, i32, i32, vp, i32, f32,
+                                         i32, vp]),
         "tk_attn_decode": (i32, [dp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp, sz, vp]),
         "tk_attn_decode_append": (i32, [dp, vp, vp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp,
                                         sz, vp]),
@@ -236,6 +238,34 @@ def tk_attn_decode_append(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_se
                                    TK_F32 if out.dtype == torch.float32 else TK_BF16, scale,
                                    _ptr(workspace), workspace.numel(), _stream(stream)),
            "tk_attn_decode_append")
+    return out
+
+
+def tk_attn_prefill_cached(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_seq_len: int, out,
+                           scale: float | None = None, causal: bool = True, stream=None):
+    """Append a chunk (k_new [B, H_kv, S, r], v_new [B, H_kv, S, d_v] bf16) at seq_lens[b]
+    and prefill its queries q [B, H_q, S, r] over the cache (query i at position
+    seq_lens[b] + i) -> out [B, H_q, S, d_v] (fp32 or bf16)."""
+    d = cache.desc
+    dev = cache.k.device
+    for t, n in ((q, "q"), (k_new, "k_new"), (v_new, "v_new")):
+        _need(t, torch.bfloat16, n, dev)
+    _need(seq_lens, torch.int32, "seq_lens", dev)
+    if out.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("out must be float32 or bfloat16")
+    _need(out, out.dtype, "out", dev)
+    S = q.shape[2]
+    if tuple(q.shape) != (d.batch, d.h_q, S, d.r) or tuple(out.shape) != (d.batch, d.h_q, S, d.d_v) \
+            or tuple(k_new.shape) != (d.batch, d.h_kv, S, d.r) \
+            or tuple(v_new.shape) != (d.batch, d.h_kv, S, d.d_v):
+        raise ValueError("q / k_new / v_new / out shapes do not match the cache")
+    scale = 1.0 / math.sqrt(d.r) if scale is None else float(scale)
+    L = load_library()
+    _check(L.tk_attn_prefill_cached(ctypes.byref(d), _ptr(q), _ptr(cache.k), _ptr(cache.v),
+                                    _ptr(cache.page_table), _ptr(seq_lens), _ptr(k_new), _ptr(v_new),
+                                    S, int(max_seq_len), _ptr(out),
+                                    TK_F32 if out.dtype == torch.float32 else TK_BF16, scale,
+                                    1 if causal else 0, _stream(stream)), "tk_attn_prefill_cached")
     return out
 
 

@@ -78,7 +78,11 @@ def causal_pairs(seq: int) -> int:
 
 
 def prefill_flops(batch: int, h_q: int, seq: int, r: int, d_v: int,
-                  causal: bool = True) -> int:
-    """Attention FLOPs of prefill: 2 * (r + d_v) per unmasked pair."""
-    pairs = causal_pairs(seq) if causal else seq * seq
+                  causal: bool = True, cached: int = 0) -> int:
+    """Attention FLOPs of prefill: 2 * (r + d_v) per unmasked pair.  With `cached`
+    tokens before the chunk, query i sees cached + i + 1 keys (causal)."""
+    if causal:
+        pairs = cached * seq + causal_pairs(seq)
+    else:
+        pairs = (cached + seq) * seq
     return batch * h_q * pairs * 2 * (r + d_v)

@@ -82,8 +82,8 @@ cudaError_t launch_append(const AppendParams& p, cudaStream_t stream, int* unsup
 
 struct PrefillParams {
   const void* q;  // bf16 [B][Hq][S][R]
-  const void* k;  // bf16 [B][Hkv][S][R]
-  const void* v;  // bf16 [B][Hkv][S][DV]
+  const void* k;  // bf16 [B][Hkv][S][R], or the cache / pool (cached mode)
+  const void* v;  // bf16 [B][Hkv][S][DV], or the cache / pool (cached mode)
   void* out;      // [B][Hq][S][DV]
   int out_f32;
   int* err;
@@ -92,6 +92,14 @@ struct PrefillParams {
   float scale_log2;
   int num_sms;
   int head_group;  // (b, h) pairs per L2 group, set by the launcher
+  // cached mode (a chunk of S queries after seq_lens[b] cached tokens):
+  // query i of sequence b sits at position seq_lens[b] + i and the keys are
+  // the cache's first seq_lens[b] + S tokens (bottom-right causal)
+  const int32_t* seq_lens;  // nullptr: plain prefill (no cache)
+  const int32_t* page_table;
+  int capacity;             // contiguous cache rows per (b, g)
+  int page_size, page_shift, num_pages, max_pages;  // paged (page_size 0 = contiguous)
+  int kv_limit;             // bound of seq_lens[b] + S
 };
 
 cudaError_t launch_prefill(const PrefillParams& p, cudaStream_t stream, int* unsupported);

@@ -345,9 +345,24 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   const int kv_plane = b * p.Hkv + h / (p.Hq / p.Hkv);
   const int qa = 2 * tp, qb = 2 * tp + 1;
   const bool has_b = qb < n_qt;
-  const int n_kv_all = (p.S + kBN - 1) / kBN;
-  const int n_a = p.causal ? min(n_kv_all, qa + 1) : n_kv_all;
-  const int n_b = has_b ? (p.causal ? min(n_kv_all, qb + 1) : n_kv_all) : 0;
+  // keys: the sequence's first kv_len cache tokens; query row i sits at position L0 + i
+  int L0 = 0;
+  if (p.seq_lens) {
+    L0 = p.seq_lens[b];
+    if (L0 < 0 || L0 > p.kv_limit - p.S) {
+      if (tid == 0) record_error(p.err, TK_DEVERR_INDEX);
+      L0 = L0 < 0 ? 0 : p.kv_limit - p.S;
+    }
+  }
+  const int kv_len = L0 + p.S;
+  const int n_kv_all = (kv_len + kBN - 1) / kBN;
+  // a causal query tile needs the kv tiles up to its last row's position
+  auto tiles_for = [&](int qt) {
+    const int last = L0 + min(qt * kBM + kBM, p.S) - 1;
+    return p.causal ? min(n_kv_all, last / kBN + 1) : n_kv_all;
+  };
+  const int n_a = tiles_for(qa);
+  const int n_b = has_b ? tiles_for(qb) : 0;
   const int n_kv = max(n_a, n_b);
 
   if (tid == 0) {
@@ -374,6 +389,12 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
 
   if (warp == 8) {
     // ------------------------------------------------------------------ TMA producer
+    // K/V maps are [planes][rows][width]: plane b*Hkv + g with rows = S (plain) or
+    // the capacity (contiguous cache), or plane page*Hkv + g with rows = page_size
+    // (paged); a 128-key tile is one box, or 128 / page_size boxes from several pages.
+    const int g = h / (p.Hq / p.Hkv);
+    const int bps = (p.page_size == 0 || p.page_size >= kBN) ? kBN : p.page_size;
+    const int nsub = kBN / bps;
     if (lane == 0) {
       prefetch_map(&maps.q);
       prefetch_map(&maps.k);
@@ -383,17 +404,46 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
         for (int i = 0; i < C::QK_NBOX; ++i)
           tma_load_3d(smem + C::OFF_Q + x * C::QBA + i * C::QK_BOXB, &maps.q, i * C::QK_BOX,
                       (qa + x) * kBM, bh, q_full);
-      for (int j = 0; j < n_kv; ++j) {
-        const int st = j % NST;
-        if (j >= NST && !mbar_wait(&kv_empty[st], ((j / NST) - 1) & 1, p.err)) break;
+    }
+    for (int j = 0; j < n_kv; ++j) {
+      const int st = j % NST;
+      int okw = 1;
+      if (j >= NST && lane == 0) okw = mbar_wait(&kv_empty[st], ((j / NST) - 1) & 1, p.err);
+      if (!__shfl_sync(0xffffffffu, okw, 0)) break;
+      // lane s < nsub finds the plane and first row of sub-box s
+      int plane = kv_plane, row = j * kBN;
+      if (p.page_size != 0) {
+        const int t = j * kBN + lane * bps;
+        int page = -1;  // keys past the sequence's pages read the zero fill
+        if (lane < nsub && t < kv_len) {
+          page = p.page_table[static_cast<long long>(b) * p.max_pages + (t >> p.page_shift)];
+          if (page < 0 || page >= p.num_pages) {
+            record_error(p.err, TK_DEVERR_INDEX);
+            page = 0;
+          }
+        }
+        plane = page < 0 ? -1 : page * p.Hkv + g;
+        row = t & (p.page_size - 1);
+      }
+      int planes[kBN / 16], rows[kBN / 16];
+#pragma unroll
+      for (int s2 = 0; s2 < kBN / 16; ++s2) {
+        planes[s2] = __shfl_sync(0xffffffffu, plane, s2);
+        rows[s2] = __shfl_sync(0xffffffffu, row, s2);
+      }
+      if (lane == 0) {
         unsigned char* sk = smem + C::OFF_K + st * C::STAGE;
         unsigned char* sv = sk + C::KBA;
         mbar_arrive_expect_tx(&k_full[st], C::KB);
-        for (int i = 0; i < C::QK_NBOX; ++i)
-          tma_load_3d(sk + i * C::QK_BOXB, &maps.k, i * C::QK_BOX, j * kBN, kv_plane, &k_full[st]);
+        for (int s2 = 0; s2 < nsub; ++s2)
+          for (int i = 0; i < C::QK_NBOX; ++i)
+            tma_load_3d(sk + i * C::QK_BOXB + s2 * bps * C::QK_SW, &maps.k, i * C::QK_BOX,
+                        rows[s2], planes[s2], &k_full[st]);
         mbar_arrive_expect_tx(&v_full[st], C::VB);
-        for (int i = 0; i < C::V_NBOX; ++i)
-          tma_load_3d(sv + i * C::V_BOXB, &maps.v, i * 64, j * kBN, kv_plane, &v_full[st]);
+        for (int s2 = 0; s2 < nsub; ++s2)
+          for (int i = 0; i < C::V_NBOX; ++i)
+            tma_load_3d(sv + i * C::V_BOXB + s2 * bps * 128, &maps.v, i * 64, rows[s2], planes[s2],
+                        &v_full[st]);
       }
     }
   } else if (warp == 9) {
@@ -465,7 +515,8 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
     const int qt = x == 0 ? qa : qb;
     const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
     const uint32_t tS = tmem + x * 128, tO = tmem + 256 + x * 128;
-    const int row = qt * kBM + (tid & 127);    // query position of this thread
+    const int row = qt * kBM + (tid & 127);    // query row of this thread in the chunk
+    const int pos = L0 + row;                  // its position among the keys
     const float sl2 = p.scale_log2;
     float m_used = -INFINITY, l = 0.f;
     bool ok = nx > 0;
@@ -474,8 +525,8 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
       tc_fence_after();
       const int kv0 = j * kBN;
-      const bool masked = (p.causal && kv0 + kBN - 1 > qt * kBM) || (kv0 + kBN > p.S);
-      const int lim = min(p.S - kv0, p.causal ? row - kv0 + 1 : kBN);  // visible columns
+      const bool masked = (p.causal && kv0 + kBN - 1 > L0 + qt * kBM) || (kv0 + kBN > kv_len);
+      const int lim = min(kv_len - kv0, p.causal ? pos - kv0 + 1 : kBN);  // visible columns
       // the whole S row of this thread: 128 fp32 scores
       uint32_t v[128];
       tmem_ld128(tS + lane_off, v);
@@ -589,16 +640,16 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// 3-D bf16 map over [planes][rows][inner] with a (box_inner x 128 x 1) box.
+// 3-D bf16 map over [planes][rows][inner] with a (box_inner x box_rows x 1) box.
 bool make_map(CUtensorMap* m, const void* base, int inner, int rows, int planes, int box_inner,
-              int swizzle_bytes) {
+              int box_rows, int swizzle_bytes) {
   auto enc = encode_fn();
   if (!enc) return false;
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows),
                         static_cast<cuuint64_t>(planes)};
   cuuint64_t strides[2] = {static_cast<cuuint64_t>(inner) * 2,
                            static_cast<cuuint64_t>(inner) * rows * 2};
-  cuuint32_t box[3] = {static_cast<cuuint32_t>(box_inner), 128, 1};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(box_inner), static_cast<cuuint32_t>(box_rows), 1};
   cuuint32_t estr[3] = {1, 1, 1};
   CUtensorMapSwizzle sw = swizzle_bytes == 32   ? CU_TENSOR_MAP_SWIZZLE_32B
                           : swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
@@ -612,9 +663,19 @@ template <int R, int DV>
 cudaError_t launch_t(const PrefillParams& p, cudaStream_t stream) {
   using C = PCfg<R, DV>;
   Maps maps;
-  if (!make_map(&maps.q, p.q, R, p.S, p.B * p.Hq, C::QK_BOX, C::QK_SW) ||
-      !make_map(&maps.k, p.k, R, p.S, p.B * p.Hkv, C::QK_BOX, C::QK_SW) ||
-      !make_map(&maps.v, p.v, DV, p.S, p.B * p.Hkv, 64, 128))
+  // K / V: [B*Hkv][S] inputs, a contiguous cache [B*Hkv][capacity] or a paged
+  // pool [num_pages*Hkv][page_size] (boxes of min(page_size, 128) rows)
+  int kv_rows = p.S, kv_planes = p.B * p.Hkv, box_rows = kBM;
+  if (p.seq_lens && p.page_size == 0) {
+    kv_rows = p.capacity;
+  } else if (p.seq_lens) {
+    kv_rows = p.page_size;
+    kv_planes = p.num_pages * p.Hkv;
+    box_rows = std::min(p.page_size, kBN);
+  }
+  if (!make_map(&maps.q, p.q, R, p.S, p.B * p.Hq, C::QK_BOX, kBM, C::QK_SW) ||
+      !make_map(&maps.k, p.k, R, kv_rows, kv_planes, C::QK_BOX, box_rows, C::QK_SW) ||
+      !make_map(&maps.v, p.v, DV, kv_rows, kv_planes, 64, box_rows, 128))
     return cudaErrorInvalidValue;
   auto kern = prefill_kernel<R, DV>;
   const int smem = C::SMEM;
@@ -624,7 +685,7 @@ cudaError_t launch_t(const PrefillParams& p, cudaStream_t stream) {
   const long grid = (n_qt + 1) / 2 * p.B * p.Hq;  // one CTA per query tile pair
   PrefillParams pp = p;
   // about 48 MB of K/V per head group
-  const long head_bytes = static_cast<long>(p.S) * (R + DV) * 2;
+  const long head_bytes = static_cast<long>(p.seq_lens ? p.kv_limit : p.S) * (R + DV) * 2;
   pp.head_group = static_cast<int>(std::max(1L, std::min<long>(p.B * p.Hq, (48L << 20) / head_bytes)));
   if (grid > 0x7fffffffL) return cudaErrorInvalidConfiguration;
   kern<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(maps, pp);

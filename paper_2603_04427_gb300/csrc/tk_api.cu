@@ -3,6 +3,7 @@
 // to the kernels.  Nothing here allocates device memory.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -180,6 +181,72 @@ tk_status tk_attn_prefill(const void* q, const void* k, const void* v, void* out
   int uns = 0;
   cudaError_t e = tk::launch_prefill(p, static_cast<cudaStream_t>(stream), &uns);
   if (uns) return fail(TK_ERR_UNSUPPORTED, "prefill: no kernel for r=%d d_v=%d", r, d_v);
+  if (e != cudaSuccess) return cuda_fail(e, "prefill launch");
+  return TK_OK;
+}
+
+tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void* k_cache,
+                                 void* v_cache, const int32_t* page_table,
+                                 const int32_t* seq_lens, const void* k_new, const void* v_new,
+                                 int32_t seq, int32_t max_seq_len, void* out, int32_t out_dtype,
+                                 float scale, int32_t causal, void* stream) {
+  tk_status s = check_desc(desc);
+  if (s != TK_OK) return s;
+  if (desc->k_dtype != TK_BF16)
+    return fail(TK_ERR_UNSUPPORTED, "prefill over a cache needs bf16 keys (k_dtype=%d)",
+                desc->k_dtype);
+  if (seq < 0 || max_seq_len < seq)
+    return fail(TK_ERR_INVALID_ARG, "seq=%d max_seq_len=%d", seq, max_seq_len);
+  if (out_dtype != TK_BF16 && out_dtype != TK_F32)
+    return fail(TK_ERR_UNSUPPORTED, "out_dtype=%d (supported: TK_BF16, TK_F32)", out_dtype);
+  if (!std::isfinite(scale) || !(scale > 0.f))
+    return fail(TK_ERR_INVALID_ARG, "prefill scale must be finite and positive");
+  if (desc->batch == 0 || seq == 0) return TK_OK;
+  if ((s = check_cache_ptrs(desc, k_cache, v_cache, nullptr, page_table)) != TK_OK) return s;
+  if (!q || !out || !seq_lens || !k_new || !v_new)
+    return fail(TK_ERR_INVALID_ARG, "q / out / seq_lens / k_new / v_new is NULL");
+  if (!aligned16(q) || !aligned16(out) || !aligned16(k_new) || !aligned16(v_new))
+    return fail(TK_ERR_INVALID_ARG, "q / out / k_new / v_new must be 16-byte aligned");
+  DeviceInfo* dev;
+  if ((s = device_info(&dev)) != TK_OK) return s;
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // 1. the chunk's keys and values into the cache at seq_lens[b]
+  tk::AppendParams a{};
+  a.k = k_cache; a.v = v_cache; a.k_scale = nullptr; a.page_table = page_table;
+  a.seq_lens = seq_lens; a.k_new = k_new; a.v_new = v_new; a.err = dev->err;
+  a.B = desc->batch; a.Hkv = desc->h_kv; a.R = desc->r; a.DV = desc->d_v; a.T = seq;
+  a.k_fmt = 0;
+  a.capacity = desc->capacity;
+  a.page_size = desc->page_size;
+  a.page_shift = desc->page_size ? log2i(desc->page_size) : 0;
+  a.num_pages = desc->num_pages; a.max_pages = desc->max_pages_per_seq;
+  int uns = 0;
+  cudaError_t e = tk::launch_append(a, st, &uns);
+  if (uns) return fail(TK_ERR_UNSUPPORTED, "append: no kernel for r=%d d_v=%d", desc->r, desc->d_v);
+  if (e != cudaSuccess) return cuda_fail(e, "append launch");
+  // 2. the chunk's queries over the cache's first seq_lens[b] + seq tokens
+  tk::PrefillParams p{};
+  p.q = q; p.k = k_cache; p.v = v_cache; p.out = out; p.out_f32 = out_dtype == TK_F32;
+  p.err = dev->err;
+  p.B = desc->batch; p.Hq = desc->h_q; p.Hkv = desc->h_kv; p.S = seq; p.R = desc->r;
+  p.DV = desc->d_v;
+  p.causal = causal != 0;
+  p.scale_log2 = scale * 1.4426950408889634f;
+  p.num_sms = dev->num_sms;
+  p.seq_lens = seq_lens;
+  p.page_table = page_table;
+  p.capacity = desc->capacity;
+  p.page_size = desc->page_size;
+  p.page_shift = a.page_shift;
+  p.num_pages = desc->num_pages;
+  p.max_pages = desc->max_pages_per_seq;
+  const int cache_tokens = desc->page_size ? desc->max_pages_per_seq * desc->page_size
+                                           : desc->capacity;
+  p.kv_limit = std::min(max_seq_len, cache_tokens);
+  if (p.kv_limit < seq)
+    return fail(TK_ERR_INVALID_ARG, "seq=%d does not fit the cache (%d tokens)", seq, p.kv_limit);
+  e = tk::launch_prefill(p, st, &uns);
+  if (uns) return fail(TK_ERR_UNSUPPORTED, "prefill: no kernel for r=%d d_v=%d", desc->r, desc->d_v);
   if (e != cudaSuccess) return cuda_fail(e, "prefill launch");
   return TK_OK;
 }

@@ -30,6 +30,7 @@ class Workload:
     seed: int = 1000
     notes: str = ""
     r_sweep: tuple = field(default_factory=tuple)
+    cached: int = 0       # prefill of a chunk after this many cached tokens
 
     def as_config(self) -> dict:
         d = {"workload": self.name, "batch": self.batch, "h_q": self.h_q, "h_kv": self.h_kv,
@@ -40,6 +41,8 @@ class Workload:
             d["seq_range"] = list(self.seq_range)
         if self.page_size:
             d["page_size"] = self.page_size
+        if self.cached:
+            d["cached"] = self.cached
         d["k_dtype"] = "int8" if self.k_int8 else "bf16"
         return d
 
@@ -51,6 +54,10 @@ MISTRAL_GQA_DECODE = Workload("mistral7b_gqa_decode_b16_ctx4096", "decode", 16, 
                               seq=4096, seed=1001)
 MHA7B_PREFILL = Workload("mha7b_causal_prefill_b2_s8192", "prefill", 2, 32, 32, 32, 128, seq=8192,
                          seed=1002, notes="bf16 output")
+# Chunked prefill (a serving engine's prompt chunk): 4096 new tokens of the 7B
+# shape after 4096 cached ones, the keys read back from a contiguous cache.
+CHUNKED_PREFILL = Workload("mha7b_chunked_prefill_b2_4096_after_4096", "prefill", 2, 32, 32, 32, 128,
+                           seq=4096, cached=4096, seed=1006, notes="bf16 output")
 PAGED_LONG_DECODE = Workload("paged_decode_b4_ctx64k_128k", "decode", 4, 32, 8, 32, 128,
                              seq_range=(65536, 131072), page_size=64, seed=1003)
 INT8_DECODE = Workload("int8_key_decode_b64_ctx32768", "decode", 64, 32, 8, 32, 128, seq=32768,

@@ -125,6 +125,23 @@ def test_decode_append_validation(lib):
     assert "k_scale" in tb.tk_last_error()
 
 
+def test_prefill_cached_validation(lib):
+    P = lib.tk_attn_prefill_cached
+    d = _desc()
+    args = (FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, 64, 256, FAKE, tb.TK_BF16, 0.1, 1, None)
+    d8 = _desc(k_dtype=tb.TK_I8)
+    assert P(ctypes.byref(d8), *args) == tb.TK_ERR_UNSUPPORTED
+    assert "bf16 keys" in tb.tk_last_error()
+    assert P(ctypes.byref(d), FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, 64, 32, FAKE, tb.TK_BF16,
+             0.1, 1, None) == tb.TK_ERR_INVALID_ARG            # max_seq_len < seq
+    assert P(ctypes.byref(d), None, FAKE, FAKE, None, FAKE, FAKE, FAKE, 64, 256, FAKE, tb.TK_BF16,
+             0.1, 1, None) == tb.TK_ERR_INVALID_ARG            # q is NULL
+    assert P(ctypes.byref(d), FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, 64, 256, FAKE, tb.TK_BF16,
+             -1.0, 1, None) == tb.TK_ERR_INVALID_ARG           # scale <= 0
+    assert P(ctypes.byref(d), None, None, None, None, None, None, None, 0, 0, None, tb.TK_BF16,
+             0.1, 1, None) == tb.TK_OK                          # empty chunk: no-op
+
+
 def test_prefill_validation(lib):
     P = lib.tk_attn_prefill
     assert P(FAKE, FAKE, FAKE, FAKE, tb.TK_BF16, 2, 6, 4, 128, 32, 128, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG

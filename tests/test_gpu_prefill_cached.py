@@ -1,0 +1,129 @@
+"""tk_attn_prefill_cached: a chunk of queries over a cached context, on the GPU.
+
+The chunk's keys and values land in the cache (bit-exact); its queries at
+positions seq_lens[b] + i attend to the cache's first seq_lens[b] + i + 1
+tokens (end-aligned causal) and match the fp64 oracle; paged caches give the
+same bits as a contiguous one, and an empty context gives the plain prefill
+bit for bit.  A 7B-shaped chunk (4096 new tokens after 4096 cached) is
+checked on sampled rows.
+"""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from _helpers import f64, parity, parity_bf16, require_gpu
+from oracle import attention as oa
+from paper_2603_04427_gb300 import binding as tb
+from paper_2603_04427_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+
+
+def _setup(B, hq, hkv, r, dv, L0, S, seed, ps=0):
+    cap = (max(L0) + S + 15) // 16 * 16
+    n = [l0 + S for l0 in L0]
+    if ps:
+        table, n_pages = inputs.paged_layout(n, ps, seed=seed, extra_pages=2)
+        cache = tb.ThinKeyCache.allocate(B, hq, hkv, r, dv, page_size=ps, num_pages=n_pages,
+                                         page_table=table)
+    else:
+        cache = tb.ThinKeyCache.allocate(B, hq, hkv, r, dv, capacity=cap)
+    T = max(L0)
+    kc = inputs.normal_bf16((B, hkv, max(T, 1), r), seed, device="cuda")
+    vc = inputs.normal_bf16((B, hkv, max(T, 1), dv), seed + 1, device="cuda")
+    zero = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for b, l0 in enumerate(L0):   # the cached context of each sequence
+        if l0:
+            d = cache.desc
+            one = tb.ThinKeyCache(tb.tk_cache_desc(1, hq, hkv, r, dv, d.capacity, d.page_size,
+                                                   d.num_pages, d.max_pages_per_seq, d.k_dtype),
+                                  cache.k if ps else cache.k[b:b + 1], cache.v if ps else cache.v[b:b + 1],
+                                  None, cache.page_table[b:b + 1].contiguous() if ps else None)
+            tb.tk_kv_append(one, kc[b:b + 1, :, :l0].contiguous(), vc[b:b + 1, :, :l0].contiguous(), zero)
+    q = inputs.normal_bf16((B, hq, S, r), seed + 2, device="cuda")
+    kn = inputs.normal_bf16((B, hkv, S, r), seed + 3, device="cuda")
+    vn = inputs.normal_bf16((B, hkv, S, dv), seed + 4, device="cuda")
+    # the whole context per sequence, for the oracle
+    K = torch.zeros(B, hkv, max(n), r, dtype=torch.bfloat16, device="cuda")
+    V = torch.zeros(B, hkv, max(n), dv, dtype=torch.bfloat16, device="cuda")
+    for b, l0 in enumerate(L0):
+        K[b, :, :l0], V[b, :, :l0] = kc[b, :, :l0], vc[b, :, :l0]
+        K[b, :, l0:l0 + S], V[b, :, l0:l0 + S] = kn[b], vn[b]
+    return cache, q, kn, vn, K, V, max(n)
+
+
+def _run(cache, q, kn, vn, L0, max_len, dtype=torch.float32, causal=True):
+    B, hq, S, _ = q.shape
+    out = torch.full((B, hq, S, cache.desc.d_v), float("nan"), dtype=dtype, device="cuda")
+    sl = torch.tensor(L0, dtype=torch.int32, device="cuda")
+    tb.tk_attn_prefill_cached(cache, q, kn, vn, sl, max_len, out, causal=causal)
+    assert tb.tk_get_device_error() == 0
+    return out
+
+
+@pytest.mark.parametrize("r,dv", [(32, 128), (64, 64), (16, 128), (128, 128)])
+def test_cached_prefill_matches_oracle(r, dv):
+    require_gpu()
+    B, hq, hkv, S = 3, 8, 2, 300
+    L0 = [0, 100, 777]
+    cache, q, kn, vn, K, V, n = _setup(B, hq, hkv, r, dv, L0, S, seed=10 + r)
+    out = _run(cache, q, kn, vn, L0, n)
+    ref = oa.attention_prefill_cached(f64(q), f64(K), f64(V), L0, 1 / math.sqrt(r))
+    parity(f64(out), ref, what=f"cached prefill r={r} dv={dv}")
+    for b, l0 in enumerate(L0):   # the chunk is in the cache
+        assert torch.equal(cache.k[b, :, l0:l0 + S], kn[b])
+        assert torch.equal(cache.v[b, :, l0:l0 + S], vn[b])
+
+
+def test_cached_prefill_non_causal_and_bf16_out():
+    require_gpu()
+    B, hq, hkv, r, dv, S = 2, 4, 4, 32, 128, 200
+    L0 = [64, 333]
+    cache, q, kn, vn, K, V, n = _setup(B, hq, hkv, r, dv, L0, S, seed=3)
+    out = _run(cache, q, kn, vn, L0, n, dtype=torch.bfloat16, causal=False)
+    ref = oa.attention_prefill_cached(f64(q), f64(K), f64(V), L0, 1 / math.sqrt(r), causal=False)
+    parity_bf16(f64(out), ref, what="cached prefill, full attention, bf16 out")
+
+
+@pytest.mark.parametrize("ps", [16, 64, 128, 256])
+def test_cached_prefill_paged_equals_contiguous_bitwise(ps):
+    require_gpu()
+    B, hq, hkv, r, dv, S = 3, 8, 2, 32, 128, 257
+    L0 = [5, 130, 640]
+    a = _setup(B, hq, hkv, r, dv, L0, S, seed=21)
+    p = _setup(B, hq, hkv, r, dv, L0, S, seed=21, ps=ps)
+    out_a = _run(*a[:4], L0, a[6])
+    out_p = _run(*p[:4], L0, p[6])
+    assert torch.equal(out_a, out_p)
+
+
+def test_empty_context_equals_plain_prefill():
+    require_gpu()
+    B, hq, hkv, r, dv, S = 2, 8, 4, 32, 128, 390
+    L0 = [0, 0]
+    cache, q, kn, vn, _, _, n = _setup(B, hq, hkv, r, dv, L0, S, seed=31)
+    out = _run(cache, q, kn, vn, L0, n)
+    plain = torch.empty_like(out)
+    tb.tk_attn_prefill(q, kn, vn, plain)
+    assert torch.equal(out, plain)
+
+
+def test_7b_chunk_after_4096_cached_sampled():
+    """B=2, H=32, r=32, d_v=128: 4096 new tokens after 4096 cached, bf16 out, sampled rows."""
+    require_gpu()
+    B, H, r, dv, S = 2, 32, 32, 128, 4096
+    L0 = [4096, 4096]
+    cache, q, kn, vn, K, V, n = _setup(B, H, H, r, dv, L0, S, seed=1005)
+    out = _run(cache, q, kn, vn, L0, n, dtype=torch.bfloat16)
+    rng = np.random.default_rng(5)
+    got, ref = [], []
+    for b, h, i in [(int(rng.integers(B)), int(rng.integers(H)), int(i)) for i in
+                    list(rng.integers(0, S, 40)) + [0, 127, 128, 4095]]:
+        p = L0[b] + i
+        ref.append(oa.attention_head(f64(q[b, h, i])[None], f64(K[b, h, :p + 1]),
+                                     f64(V[b, h, :p + 1]), 1 / math.sqrt(r))[0])
+        got.append(f64(out[b, h, i]))
+    parity_bf16(np.stack(got), np.stack(ref), what="7b cached chunk sampled")
