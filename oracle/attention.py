@@ -130,6 +130,49 @@ def attention_prefill_cached(q, k, v, seq_lens, scale: float, causal: bool = Tru
     return out
 
 
+def attention_backward(q, k, v, d_out, scale: float, causal: bool = True):
+    """Gradients of prefill attention (Eqs. 1-4) for a loss with dL/d(out) = d_out.
+
+    q: [B, H_q, S, r], k: [B, H_kv, S, r], v: [B, H_kv, S, d_v], d_out: [B, H_q, S, d_v].
+    Per head, with s = scale q k^T (masked), p = softmax(s) row-wise, out = p v:
+        dv = p^T d_out,  dp = d_out v^T,  ds = p * (dp - rowsum(dp * p)),
+        dq = scale ds k,  dk = scale ds^T q
+    (the softmax Jacobian diag(p) - p p^T applied row by row); a kv head's dk and dv
+    sum the contributions of its G query heads.  Returns (dq, dk, dv) float64.
+    """
+    q, k, v, d_out = (np.asarray(x, dtype=np.float64) for x in (q, k, v, d_out))
+    B, h_q, S, _ = q.shape
+    h_kv = k.shape[1]
+    dq, dk, dv = np.zeros_like(q), np.zeros_like(k), np.zeros_like(v)
+    for b in range(B):
+        for h in range(h_q):
+            g = _kv_head(h, h_q, h_kv)
+            _, p = attention_head(q[b, h], k[b, g], v[b, g], scale,
+                                  causal_offset=0 if causal else None, return_weights=True)
+            dv[b, g] += p.T @ d_out[b, h]
+            dp = d_out[b, h] @ v[b, g].T
+            ds = p * (dp - np.sum(dp * p, axis=1, keepdims=True))
+            dq[b, h] = scale * (ds @ k[b, g])
+            dk[b, g] += scale * (ds.T @ q[b, h])
+    return dq, dk, dv
+
+
+def logsumexp_rows(q, k, scale: float, causal: bool = True) -> np.ndarray:
+    """Natural-log logsumexp of each row's scaled (masked) scores: [B, H_q, S]."""
+    q, k = np.asarray(q, dtype=np.float64), np.asarray(k, dtype=np.float64)
+    B, h_q, S, _ = q.shape
+    h_kv = k.shape[1]
+    out = np.zeros((B, h_q, S))
+    for b in range(B):
+        for h in range(h_q):
+            s = scale * (q[b, h] @ k[b, _kv_head(h, h_q, h_kv)].T)
+            if causal:
+                s = np.where(np.arange(S)[None, :] <= np.arange(S)[:, None], s, -np.inf)
+            m = s.max(axis=1)
+            out[b, h] = m + np.log(np.exp(s - m[:, None]).sum(axis=1))
+    return out
+
+
 def attention_prefill_rows(q, k, v, scale: float, rows, causal: bool = True) -> np.ndarray:
     """Selected output rows of ``attention_prefill``, each computed on its own.
 

@@ -277,6 +277,55 @@ def test_cached_prefill_brute_force():
         np.testing.assert_allclose(got[0, 0, i], want, rtol=1e-12, atol=1e-14)
 
 
+# ---------------------------------------------------------------- backward
+
+@pytest.mark.parametrize("causal", [True, False])
+def test_backward_matches_torch_autograd(causal):
+    """Independent route: torch autograd through an fp64 softmax attention."""
+    B, hq, hkv, S, r, dv = 2, 4, 2, 11, 6, 5
+    q, k, v, do = _rand(B, hq, S, r), _rand(B, hkv, S, r), _rand(B, hkv, S, dv), _rand(B, hq, S, dv)
+    dq, dk, dv_ = oa.attention_backward(q, k, v, do, 0.37, causal)
+    tq, tk, tv = (torch.tensor(x, requires_grad=True) for x in (q, k, v))
+    G = hq // hkv
+    kk, vv = tk.repeat_interleave(G, dim=1), tv.repeat_interleave(G, dim=1)
+    s = 0.37 * tq @ kk.transpose(-1, -2)
+    if causal:
+        s = s.masked_fill(torch.triu(torch.ones(S, S, dtype=torch.bool), 1), float("-inf"))
+    out = torch.softmax(s, dim=-1) @ vv
+    (out * torch.tensor(do)).sum().backward()
+    np.testing.assert_allclose(dq, tq.grad.numpy(), rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(dk, tk.grad.numpy(), rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(dv_, tv.grad.numpy(), rtol=1e-11, atol=1e-12)
+
+
+def test_backward_finite_differences():
+    B, hq, hkv, S, r, dv = 1, 2, 1, 5, 3, 2
+    q, k, v, do = _rand(B, hq, S, r), _rand(B, hkv, S, r), _rand(B, hkv, S, dv), _rand(B, hq, S, dv)
+    grads = oa.attention_backward(q, k, v, do, 0.8)
+
+    def loss(qq, kk, vv):
+        return float(np.sum(oa.attention_prefill(qq, kk, vv, 0.8) * do))
+    eps = 1e-6
+    for idx, (x, gx) in enumerate(zip((q, k, v), grads)):
+        for pos in [(0, 0, 2, 1), (0, hq - 1 if idx == 0 else 0, 4, 0), (0, 0, 0, dv - 1 if idx == 2 else 0)]:
+            xp, xm = x.copy(), x.copy()
+            xp[pos] += eps
+            xm[pos] -= eps
+            args_p = [q, k, v]; args_p[idx] = xp
+            args_m = [q, k, v]; args_m[idx] = xm
+            num = (loss(*args_p) - loss(*args_m)) / (2 * eps)
+            assert abs(num - gx[pos]) <= 1e-7 * max(1.0, abs(num))
+
+
+def test_logsumexp_rows():
+    q, k = _rand(1, 2, 7, 4), _rand(1, 1, 7, 4)
+    lse = oa.logsumexp_rows(q, k, 0.5)
+    for h in range(2):
+        for i in range(7):
+            s = 0.5 * (q[0, h, i] @ k[0, 0, :i + 1].T)
+            assert lse[0, h, i] == pytest.approx(math.log(math.fsum(math.exp(x) for x in s)), rel=1e-13)
+
+
 # ---------------------------------------------------------------- int8 keys
 
 def test_quantiser_ties_round_to_even():
