@@ -377,6 +377,35 @@ def measure_chunked_prefill(w, iters, device, torch):
             "cached": L0, "launches": 2}
 
 
+def measure_backward(w, iters, device, torch):
+    """Training backward of the causal prefill shape (tk_attn_backward: the D / dQ-zeroing
+    pass and the gradient kernel), from a tk_attn_forward of the same inputs."""
+    from paper_2603_04427_gb300 import binding as tb
+    from paper_2603_04427_gb300 import cost_model as cm
+    from paper_2603_04427_gb300 import inputs
+    B, hq, hkv, S, r, dv = w.batch, w.h_q, w.h_kv, w.seq, w.r, w.d_v
+    q = inputs.normal_bf16((B, hq, S, r), w.seed + 1, device=device)
+    k = inputs.normal_bf16((B, hkv, S, r), w.seed + 2, device=device)
+    v = inputs.normal_bf16((B, hkv, S, dv), w.seed + 3, device=device)
+    do = inputs.normal_bf16((B, hq, S, dv), w.seed + 4, device=device)
+    out = torch.empty(B, hq, S, dv, dtype=torch.bfloat16, device=device)
+    lse = torch.empty(B, hq, S, dtype=torch.float32, device=device)
+    tb.tk_attn_forward(q, k, v, out, lse)
+    dq = torch.empty(B, hq, S, r, dtype=torch.float32, device=device)
+    dk = torch.empty(B, hkv, S, r, dtype=torch.float32, device=device)
+    dvv = torch.empty(B, hkv, S, dv, dtype=torch.float32, device=device)
+    ws = torch.empty(int(tb.load_library().tk_backward_workspace_size(B, hq, S)), dtype=torch.uint8,
+                     device=device)
+
+    def enq(_):
+        tb.tk_attn_backward(q, k, v, out, do, lse, dq, dk, dvv, ws)
+
+    sec = graph_time(torch, enq, iters, 3, max_graph=8) / iters
+    pairs = cm.causal_pairs(S) * B * hq
+    flops = pairs * 2 * (3 * r + 2 * dv)   # S^T, dP^T, dV, dK, dQ products
+    return {"ms": sec * 1e3, "tflops": flops / sec / 1e12, "flops_per_call": flops, "launches": 2}
+
+
 def measure_gpt2_layer(w, iters, device, torch):
     """GPT-2-small layer: causal prefill of S tokens (fp32 out), append of the
     prompt's keys/values, then `decode_steps` x (append 1 token + decode)."""
@@ -492,7 +521,7 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--headline-only", action="store_true",
                     help="skip the secondary workloads and the CPU baseline")
-    ap.add_argument("--only", choices=("prefill", "chunked", "gpt2", "paged", "int8"),
+    ap.add_argument("--only", choices=("prefill", "chunked", "backward", "gpt2", "paged", "int8"),
                     help="run one secondary workload alone (for profiling) and print its result")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -524,6 +553,8 @@ def main():
         res = {"only": args.only}
         if args.only == "prefill":
             res.update(measure_prefill(wl.MHA7B_PREFILL, args.steps, device, torch))
+        elif args.only == "backward":
+            res.update(measure_backward(wl.MHA7B_PREFILL, args.steps, device, torch))
         elif args.only == "chunked":
             res.update(measure_chunked_prefill(wl.CHUNKED_PREFILL, args.steps, device, torch))
         elif args.only == "gpt2":
@@ -604,6 +635,10 @@ def main():
                       traffic=recorded_traffic("prefill", pw.name,
                                                source_hash("prefill.cu", "common.cuh")))
         extra[pw.name] = dict(pw.as_config(), **pf)
+        bw = measure_backward(pw, 10, device, torch)
+        bw.update(frac=bw["tflops"] / peaks["bf16_tflops"], peak=peaks["bf16_tflops"],
+                  peak_source=peak_src, bound="tensor", kernel="mma.sync m16n8k16")
+        extra[pw.name.replace("prefill", "backward")] = dict(pw.as_config(), **bw)
         cw = wl.CHUNKED_PREFILL
         cp = measure_chunked_prefill(cw, 20, device, torch)
         cp.update(frac=cp["tflops"] / peaks["bf16_tflops"], peak=peaks["bf16_tflops"],

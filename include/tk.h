@@ -147,6 +147,42 @@ tk_status tk_attn_prefill(const void* q, const void* k, const void* v, void* out
                           int32_t seq, int32_t r, int32_t d_v, float scale, int32_t causal,
                           void* stream);
 
+/* tk_attn_prefill that also writes, for the backward pass, each query row's
+ * natural-log logsumexp of its scaled (masked) scores,
+ * lse[b][h][i] = ln sum_j exp(scale q_i . k_j)   (float [batch][h_q][seq]).
+ * Other arguments, layouts and errors as tk_attn_prefill.                  */
+tk_status tk_attn_forward(const void* q, const void* k, const void* v, void* out, float* lse,
+                          int32_t out_dtype, int32_t batch, int32_t h_q, int32_t h_kv,
+                          int32_t seq, int32_t r, int32_t d_v, float scale, int32_t causal,
+                          void* stream);
+
+/* Bytes of workspace tk_attn_backward needs (one float per query row, rounded
+ * up); 0 for invalid arguments.                                             */
+size_t tk_backward_workspace_size(int32_t batch, int32_t h_q, int32_t seq);
+
+/* Gradients of prefill attention (the training path of thin-key attention;
+ * Section 2.1, Eqs. 1-4 differentiated).  For a loss with dL/d(out) = d_out:
+ *   dq = scale dS k,  dk = scale dS^T q,  dv = P^T d_out,
+ *   dS = P * (d_out v^T - D),  D_i = sum_c d_out_ic out_ic,  P = softmax rows,
+ * with a kv head's dk and dv summed over its h_q / h_kv query heads.
+ *   q, k, v : the forward's inputs (bf16, layouts of tk_attn_prefill)
+ *   out     : the forward's output, bf16 [batch][h_q][seq][d_v]
+ *   d_out   : bf16 [batch][h_q][seq][d_v]
+ *   lse     : the forward's row logsumexp (tk_attn_forward)
+ *   dq      : float [batch][h_q][seq][r]    (overwritten)
+ *   dk      : float [batch][h_kv][seq][r]   (overwritten)
+ *   dv      : float [batch][h_kv][seq][d_v] (overwritten)
+ *   workspace: tk_backward_workspace_size bytes, 256-byte aligned (scratch)
+ *   scale, causal: as in the forward.
+ * The products run on the tensor cores with bf16 operands (P and dS rounded
+ * to bf16) and fp32 accumulation; dq is accumulated across key tiles with
+ * fp32 atomic adds, so its low bits may vary run to run.                    */
+tk_status tk_attn_backward(const void* q, const void* k, const void* v, const void* out,
+                           const void* d_out, const float* lse, float* dq, float* dk, float* dv,
+                           void* workspace, size_t workspace_bytes, int32_t batch, int32_t h_q,
+                           int32_t h_kv, int32_t seq, int32_t r, int32_t d_v, float scale,
+                           int32_t causal, void* stream);
+
 /* Prefill of a chunk of `seq` new tokens per sequence against the cache
  * (Section 2.1, Eqs. 1-4, over a context that continues an existing one):
  * first writes the chunk's thin keys and values at positions

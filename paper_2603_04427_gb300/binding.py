@@ -22,7 +22,8 @@ TK_BF16, TK_F32, TK_I8, TK_I4 = 0, 1, 2, 3
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtk.so")
 
 EXPORTED = ("tk_kv_append", "tk_attn_prefill", "tk_decode_workspace_size", "tk_attn_decode",
-            "tk_attn_decode_append", "tk_attn_decode_noalloc", "tk_attn_prefill_cached", "tk_get_device_error", "tk_status_string", "tk_last_error",
+            "tk_attn_decode_append", "tk_attn_decode_noalloc", "tk_attn_prefill_cached",
+            "tk_attn_forward", "tk_backward_workspace_size", "tk_attn_backward", "tk_get_device_error", "tk_status_string", "tk_last_error",
             "tk_abi_version")
 
 
@@ -56,6 +57,11 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tk_kv_append": (i32, [dp, vp, vp, vp, vp, vp, vp, vp, i32, vp]),
         "tk_attn_prefill": (i32, [vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, i32, vp]),
         "tk_decode_workspace_size": (sz, [dp, i32]),
+        "tk_attn_forward": (i32, [vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32, f32, i32,
+                                  vp]),
+        "tk_backward_workspace_size": (sz, [i32, i32, i32]),
+        "tk_attn_backward": (i32, [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, i32, i32, i32, i32,
+                                   i32, i32, f32, i32, vp]),
         "tk_attn_prefill_cached": (i32, [dp, vp, vp, vp, vp, vp, vp, vp, i32, i32, vp, i32, f32,
                                          i32, vp]),
         "tk_attn_decode": (i32, [dp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp, sz, vp]),
@@ -239,6 +245,58 @@ def tk_attn_decode_append(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_se
                                    _ptr(workspace), workspace.numel(), _stream(stream)),
            "tk_attn_decode_append")
     return out
+
+
+def tk_attn_forward(q, k, v, out, lse, scale: float | None = None, causal: bool = True, stream=None):
+    """tk_attn_prefill that also writes lse [B, H_q, S] (fp32), each row's logsumexp."""
+    dev = q.device
+    for t, n in ((q, "q"), (k, "k"), (v, "v")):
+        _need(t, torch.bfloat16, n, dev)
+    _need(lse, torch.float32, "lse", dev)
+    if out.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("out must be float32 or bfloat16")
+    _need(out, out.dtype, "out", dev)
+    B, hq, S, r = q.shape
+    hkv, dv = k.shape[1], v.shape[3]
+    if tuple(k.shape) != (B, hkv, S, r) or tuple(v.shape) != (B, hkv, S, dv) or \
+            tuple(out.shape) != (B, hq, S, dv) or tuple(lse.shape) != (B, hq, S):
+        raise ValueError("q / k / v / out / lse shapes are inconsistent")
+    scale = 1.0 / math.sqrt(r) if scale is None else float(scale)
+    L = load_library()
+    _check(L.tk_attn_forward(_ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(lse),
+                             TK_F32 if out.dtype == torch.float32 else TK_BF16,
+                             B, hq, hkv, S, r, dv, scale, 1 if causal else 0, _stream(stream)),
+           "tk_attn_forward")
+    return out, lse
+
+
+def tk_attn_backward(q, k, v, out, d_out, lse, dq, dk, dv, workspace=None,
+                     scale: float | None = None, causal: bool = True, stream=None):
+    """Gradients dq [B, H_q, S, r], dk [B, H_kv, S, r], dv [B, H_kv, S, d_v] (fp32)
+    of prefill attention for dL/d(out) = d_out (bf16), from the forward's lse."""
+    dev = q.device
+    for t, n in ((q, "q"), (k, "k"), (v, "v"), (out, "out"), (d_out, "d_out")):
+        _need(t, torch.bfloat16, n, dev)
+    for t, n in ((lse, "lse"), (dq, "dq"), (dk, "dk"), (dv, "dv")):
+        _need(t, torch.float32, n, dev)
+    B, hq, S, r = q.shape
+    hkv, d_v = k.shape[1], v.shape[3]
+    if tuple(k.shape) != (B, hkv, S, r) or tuple(v.shape) != (B, hkv, S, d_v) or \
+            tuple(out.shape) != (B, hq, S, d_v) or tuple(d_out.shape) != (B, hq, S, d_v) or \
+            tuple(lse.shape) != (B, hq, S) or tuple(dq.shape) != tuple(q.shape) or \
+            tuple(dk.shape) != tuple(k.shape) or tuple(dv.shape) != tuple(v.shape):
+        raise ValueError("backward tensor shapes are inconsistent")
+    L = load_library()
+    if workspace is None:
+        workspace = torch.empty(int(L.tk_backward_workspace_size(B, hq, S)), dtype=torch.uint8,
+                                device=dev)
+    _need(workspace, torch.uint8, "workspace", dev)
+    scale = 1.0 / math.sqrt(r) if scale is None else float(scale)
+    _check(L.tk_attn_backward(_ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(d_out), _ptr(lse),
+                              _ptr(dq), _ptr(dk), _ptr(dv), _ptr(workspace), workspace.numel(),
+                              B, hq, hkv, S, r, d_v, scale, 1 if causal else 0, _stream(stream)),
+           "tk_attn_backward")
+    return dq, dk, dv
 
 
 def tk_attn_prefill_cached(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_seq_len: int, out,

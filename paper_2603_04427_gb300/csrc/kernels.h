@@ -100,7 +100,26 @@ struct PrefillParams {
   int capacity;             // contiguous cache rows per (b, g)
   int page_size, page_shift, num_pages, max_pages;  // paged (page_size 0 = contiguous)
   int kv_limit;             // bound of seq_lens[b] + S
+  float* lse;               // optional [B][Hq][S]: natural-log logsumexp of each row's scores
 };
+
+struct BackwardParams {
+  const void* q;      // bf16 [B][Hq][S][R]
+  const void* k;      // bf16 [B][Hkv][S][R]
+  const void* v;      // bf16 [B][Hkv][S][DV]
+  const void* out;    // bf16 [B][Hq][S][DV]  forward output
+  const void* d_out;  // bf16 [B][Hq][S][DV]  gradient of the loss w.r.t. out
+  const float* lse;   // [B][Hq][S] natural-log logsumexp from the forward
+  float* dq;          // fp32 [B][Hq][S][R]  (accumulated: zeroed by the preprocessing kernel)
+  float* dk;          // fp32 [B][Hkv][S][R]
+  float* dv;          // fp32 [B][Hkv][S][DV]
+  float* dsum;        // [B][Hq][S] workspace: rowsum(d_out * out)
+  int B, Hq, Hkv, S, R, DV;
+  int causal;
+  float scale;
+};
+
+cudaError_t launch_backward(const BackwardParams& p, cudaStream_t stream, int* unsupported);
 
 cudaError_t launch_prefill(const PrefillParams& p, cudaStream_t stream, int* unsupported);
 

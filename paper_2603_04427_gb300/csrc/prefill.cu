@@ -588,6 +588,9 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       const float inv = 1.f / l;
       const bool store = row < p.S;
       const size_t obase = (static_cast<size_t>(bh) * p.S + row) * DV;
+      // natural-log logsumexp of the row's scaled scores (for the backward):
+      // sum_j exp(scale s_j) = 2^m_used * l
+      if (p.lse && store) p.lse[static_cast<size_t>(bh) * p.S + row] = (m_used + log2f(l)) * 0.69314718055994531f;
 #pragma unroll
       for (int c = 0; c < DV / 32; ++c) {
         uint32_t v[32];

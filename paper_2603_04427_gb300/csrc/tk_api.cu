@@ -152,10 +152,75 @@ tk_status tk_kv_append(const tk_cache_desc* desc, void* k_cache, void* v_cache, 
   return TK_OK;
 }
 
+namespace {
+tk_status prefill_impl(const void* q, const void* k, const void* v, void* out, float* lse,
+                       int32_t out_dtype, int32_t batch, int32_t h_q, int32_t h_kv, int32_t seq,
+                       int32_t r, int32_t d_v, float scale, int32_t causal, void* stream);
+}  // namespace
+
 tk_status tk_attn_prefill(const void* q, const void* k, const void* v, void* out,
                           int32_t out_dtype, int32_t batch, int32_t h_q, int32_t h_kv,
                           int32_t seq, int32_t r, int32_t d_v, float scale, int32_t causal,
                           void* stream) {
+  return prefill_impl(q, k, v, out, nullptr, out_dtype, batch, h_q, h_kv, seq, r, d_v, scale,
+                      causal, stream);
+}
+
+tk_status tk_attn_forward(const void* q, const void* k, const void* v, void* out, float* lse,
+                          int32_t out_dtype, int32_t batch, int32_t h_q, int32_t h_kv,
+                          int32_t seq, int32_t r, int32_t d_v, float scale, int32_t causal,
+                          void* stream) {
+  if (seq > 0 && batch > 0 && !lse) return fail(TK_ERR_INVALID_ARG, "lse is NULL");
+  return prefill_impl(q, k, v, out, lse, out_dtype, batch, h_q, h_kv, seq, r, d_v, scale,
+                      causal, stream);
+}
+
+size_t tk_backward_workspace_size(int32_t batch, int32_t h_q, int32_t seq) {
+  if (batch < 0 || h_q <= 0 || seq < 0) return 0;
+  return (static_cast<size_t>(batch) * h_q * seq * 4 + 255) / 256 * 256 + 256;
+}
+
+tk_status tk_attn_backward(const void* q, const void* k, const void* v, const void* out,
+                           const void* d_out, const float* lse, float* dq, float* dk, float* dv,
+                           void* workspace, size_t workspace_bytes, int32_t batch, int32_t h_q,
+                           int32_t h_kv, int32_t seq, int32_t r, int32_t d_v, float scale,
+                           int32_t causal, void* stream) {
+  if (batch < 0 || seq < 0 || h_q <= 0 || h_kv <= 0)
+    return fail(TK_ERR_INVALID_ARG, "batch=%d seq=%d h_q=%d h_kv=%d", batch, seq, h_q, h_kv);
+  if (h_q % h_kv != 0) return fail(TK_ERR_INVALID_ARG, "h_q=%d not a multiple of h_kv=%d", h_q, h_kv);
+  if (!supported_r(r)) return fail(TK_ERR_UNSUPPORTED, "r=%d (supported: 16, 32, 64, 128)", r);
+  if (!supported_dv(d_v)) return fail(TK_ERR_UNSUPPORTED, "d_v=%d (supported: 64, 128)", d_v);
+  if (!std::isfinite(scale) || !(scale > 0.f))
+    return fail(TK_ERR_INVALID_ARG, "scale must be finite and positive");
+  if (batch == 0 || seq == 0) return TK_OK;
+  if (!q || !k || !v || !out || !d_out || !lse || !dq || !dk || !dv)
+    return fail(TK_ERR_INVALID_ARG, "a tensor pointer is NULL");
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out) || !aligned16(d_out) ||
+      !aligned16(dq) || !aligned16(dk) || !aligned16(dv))
+    return fail(TK_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  const size_t need = tk_backward_workspace_size(batch, h_q, seq);
+  if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0 || workspace_bytes < need)
+    return fail(TK_ERR_WORKSPACE, "workspace needs %zu bytes, 256-byte aligned", need);
+  DeviceInfo* dev;
+  tk_status s = device_info(&dev);
+  if (s != TK_OK) return s;
+  tk::BackwardParams p{};
+  p.q = q; p.k = k; p.v = v; p.out = out; p.d_out = d_out; p.lse = lse;
+  p.dq = dq; p.dk = dk; p.dv = dv; p.dsum = static_cast<float*>(workspace);
+  p.B = batch; p.Hq = h_q; p.Hkv = h_kv; p.S = seq; p.R = r; p.DV = d_v;
+  p.causal = causal != 0;
+  p.scale = scale;
+  int uns = 0;
+  cudaError_t e = tk::launch_backward(p, static_cast<cudaStream_t>(stream), &uns);
+  if (uns) return fail(TK_ERR_UNSUPPORTED, "backward: no kernel for r=%d d_v=%d", r, d_v);
+  if (e != cudaSuccess) return cuda_fail(e, "backward launch");
+  return TK_OK;
+}
+
+namespace {
+tk_status prefill_impl(const void* q, const void* k, const void* v, void* out, float* lse,
+                       int32_t out_dtype, int32_t batch, int32_t h_q, int32_t h_kv, int32_t seq,
+                       int32_t r, int32_t d_v, float scale, int32_t causal, void* stream) {
   if (batch < 0 || seq < 0 || h_q <= 0 || h_kv <= 0)
     return fail(TK_ERR_INVALID_ARG, "batch=%d seq=%d h_q=%d h_kv=%d", batch, seq, h_q, h_kv);
   if (h_q % h_kv != 0) return fail(TK_ERR_INVALID_ARG, "h_q=%d not a multiple of h_kv=%d", h_q, h_kv);
@@ -178,12 +243,14 @@ tk_status tk_attn_prefill(const void* q, const void* k, const void* v, void* out
   p.causal = causal != 0;
   p.scale_log2 = scale * 1.4426950408889634f;
   p.num_sms = dev->num_sms;
+  p.lse = lse;
   int uns = 0;
   cudaError_t e = tk::launch_prefill(p, static_cast<cudaStream_t>(stream), &uns);
   if (uns) return fail(TK_ERR_UNSUPPORTED, "prefill: no kernel for r=%d d_v=%d", r, d_v);
   if (e != cudaSuccess) return cuda_fail(e, "prefill launch");
   return TK_OK;
 }
+}  // namespace
 
 tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void* k_cache,
                                  void* v_cache, const int32_t* page_table,

@@ -142,6 +142,23 @@ def test_prefill_cached_validation(lib):
              0.1, 1, None) == tb.TK_OK                          # empty chunk: no-op
 
 
+def test_forward_and_backward_validation(lib):
+    F = lib.tk_attn_forward
+    assert F(FAKE, FAKE, FAKE, FAKE, None, tb.TK_BF16, 2, 4, 4, 128, 32, 128, 0.1, 1,
+             None) == tb.TK_ERR_INVALID_ARG                 # lse is NULL
+    assert lib.tk_backward_workspace_size(2, 4, 100) >= 2 * 4 * 100 * 4
+    assert lib.tk_backward_workspace_size(-1, 4, 100) == 0
+    Bw = lib.tk_attn_backward
+    base = [FAKE] * 10
+    assert Bw(*base, 1 << 20, 2, 4, 4, 128, 24, 128, 0.1, 1, None) == tb.TK_ERR_UNSUPPORTED
+    assert Bw(*base, 1 << 20, 2, 6, 4, 128, 32, 128, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG
+    assert Bw(*base, 1 << 20, 2, 4, 4, 128, 32, 128, 0.0, 1, None) == tb.TK_ERR_INVALID_ARG
+    ws_small = [FAKE] * 9 + [ctypes.c_void_p(0x10000)]
+    assert Bw(*ws_small, 16, 2, 4, 4, 128, 32, 128, 0.1, 1, None) == tb.TK_ERR_WORKSPACE
+    nulls = [FAKE] * 5 + [None] + [FAKE] * 4
+    assert Bw(*nulls, 1 << 20, 2, 4, 4, 128, 32, 128, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG
+
+
 def test_prefill_validation(lib):
     P = lib.tk_attn_prefill
     assert P(FAKE, FAKE, FAKE, FAKE, tb.TK_BF16, 2, 6, 4, 128, 32, 128, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG
