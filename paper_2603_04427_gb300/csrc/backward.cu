@@ -33,6 +33,11 @@ namespace {
 
 constexpr int kTile = 64;       // keys per CTA, queries per visit
 constexpr int kBwdThreads = 128;
+#ifndef TK_BWD_PARTQ
+#define TK_BWD_PARTQ 16
+#endif
+constexpr int kPartQ = TK_BWD_PARTQ;   // queries per step of a visit (fragments held at once)
+constexpr int kParts = kTile / kPartQ;
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& a, uint32_t& b, uint32_t& c,
                                         uint32_t& d) {
@@ -133,8 +138,11 @@ struct BCfg {
   static constexpr int OFF_BUF = OFF_V + kTile * VW;
   static constexpr int BUF_Q = 0, BUF_DO = kTile * KW, BUF_LSE = BUF_DO + kTile * VW,
                        BUF_D = BUF_LSE + kTile * 4, BUF = BUF_D + kTile * 4;
-  static constexpr int OFF_DQ = OFF_BUF + 2 * BUF;          // [64][R] fp32
-  static constexpr int SMEM = OFF_DQ + kTile * R * 4;
+  // dQ partials of one part of the queries, one buffer per warp, rows padded to R + 8
+  // floats so that a warp's 64-bit fragment stores hit 32 different banks
+  static constexpr int DQP = R + 8;
+  static constexpr int OFF_DQ = OFF_BUF + 2 * BUF;          // [4 warps][kPartQ][DQP] fp32
+  static constexpr int SMEM = OFF_DQ + 4 * kPartQ * DQP * 4;
   static_assert(SMEM <= 227 * 1024, "shared memory");
 };
 
@@ -143,7 +151,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
   using C = BCfg<R, DV>;
   extern __shared__ __align__(128) unsigned char smem[];
   const uint32_t sbase = smem_addr(smem);
-  float* dqacc = reinterpret_cast<float*>(smem + C::OFF_DQ);
+  float* dqw = reinterpret_cast<float*>(smem + C::OFF_DQ);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g8 = lane >> 2, t4 = lane & 3;          // fragment row / column pair
   const int mi = lane >> 3, rr = lane & 7;          // ldmatrix: matrix, row within it
@@ -182,7 +190,6 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
   };
   if (visits > 0) load_visit(0, 0);
   cp_async_commit();
-  for (int e = tid; e < kTile * R; e += kBwdThreads) dqacc[e] = 0.f;
 
   float dv_acc[DV / 8][4], dk_acc[R / 8][4];
 #pragma unroll
@@ -206,31 +213,31 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
     const bool diag = p.causal && i == j;
 
 #pragma unroll 1
-    for (int half = 0; half < 2; ++half) {
-      const int qb = half * 32;                     // first query (in the tile) of this half
-      float sa[4][4], dp[4][4];
+    for (int part = 0; part < kParts; ++part) {
+      const int qb = part * kPartQ;                 // first query (in the tile) of this part
+      float sa[kPartQ / 8][4], dp[kPartQ / 8][4];
 #pragma unroll
-      for (int n = 0; n < 4; ++n) sa[n][0] = sa[n][1] = sa[n][2] = sa[n][3] = dp[n][0] = dp[n][1] = dp[n][2] = dp[n][3] = 0.f;
-      // ---- S^T = K Q^T (16 keys x 32 queries), k = r
+      for (int n = 0; n < kPartQ / 8; ++n) sa[n][0] = sa[n][1] = sa[n][2] = sa[n][3] = dp[n][0] = dp[n][1] = dp[n][2] = dp[n][3] = 0.f;
+      // ---- S^T = K Q^T (16 keys x kPartQ queries), k = r
 #pragma unroll
       for (int ks = 0; ks < R / 16; ++ks) {
         uint32_t a0, a1, a2, a3;
         ldsm_x4(sbase + C::OFF_K + swz<C::KW>(krow + (mi & 1) * 8 + rr, 2 * ks + (mi >> 1)), a0, a1, a2, a3);
 #pragma unroll
-        for (int np = 0; np < 2; ++np) {
+        for (int np = 0; np < kPartQ / 16; ++np) {
           uint32_t b0, b1, b2, b3;  // queries qb+16np.. : (n-tile 2np, k lo/hi), (2np+1, k lo/hi)
           ldsm_x4(bq + swz<C::KW>(qb + 16 * np + (mi >> 1) * 8 + rr, 2 * ks + (mi & 1)), b0, b1, b2, b3);
           mma16816(sa[2 * np], a0, a1, a2, a3, b0, b1);
           mma16816(sa[2 * np + 1], a0, a1, a2, a3, b2, b3);
         }
       }
-      // ---- dP^T = V dO^T (16 keys x 32 queries), k = d_v
+      // ---- dP^T = V dO^T (16 keys x kPartQ queries), k = d_v
 #pragma unroll
       for (int ks = 0; ks < DV / 16; ++ks) {
         uint32_t a0, a1, a2, a3;
         ldsm_x4(sbase + C::OFF_V + swz<C::VW>(krow + (mi & 1) * 8 + rr, 2 * ks + (mi >> 1)), a0, a1, a2, a3);
 #pragma unroll
-        for (int np = 0; np < 2; ++np) {
+        for (int np = 0; np < kPartQ / 16; ++np) {
           uint32_t b0, b1, b2, b3;
           ldsm_x4(bdo + swz<C::VW>(qb + 16 * np + (mi >> 1) * 8 + rr, 2 * ks + (mi & 1)), b0, b1, b2, b3);
           mma16816(dp[2 * np], a0, a1, a2, a3, b0, b1);
@@ -239,7 +246,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
       }
       // ---- P^T and dS^T in the accumulator layout: (key g8 | g8+8, query 2t4 | 2t4+1)
 #pragma unroll
-      for (int n = 0; n < 4; ++n) {
+      for (int n = 0; n < kPartQ / 8; ++n) {
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const int q = qb + 8 * n + 2 * t4 + (e & 1);     // query in the tile
@@ -251,9 +258,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
         }
       }
       // A operands (16 keys x 16 queries) of P^T and dS^T for the two 16-query steps
-      uint32_t pa[2][4], da[2][4];
+      uint32_t pa[kPartQ / 16][4], da[kPartQ / 16][4];
 #pragma unroll
-      for (int kk = 0; kk < 2; ++kk) {
+      for (int kk = 0; kk < kPartQ / 16; ++kk) {
         pa[kk][0] = pack_bf16(sa[2 * kk][0], sa[2 * kk][1]);
         pa[kk][1] = pack_bf16(sa[2 * kk][2], sa[2 * kk][3]);
         pa[kk][2] = pack_bf16(sa[2 * kk + 1][0], sa[2 * kk + 1][1]);
@@ -263,9 +270,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
         da[kk][2] = pack_bf16(dp[2 * kk + 1][0], dp[2 * kk + 1][1]);
         da[kk][3] = pack_bf16(dp[2 * kk + 1][2], dp[2 * kk + 1][3]);
       }
-      // ---- dV += P^T dO (16 keys x d_v), k = 32 queries
+      // ---- dV += P^T dO (16 keys x d_v), k = kPartQ queries
 #pragma unroll
-      for (int kk = 0; kk < 2; ++kk) {
+      for (int kk = 0; kk < kPartQ / 16; ++kk) {
 #pragma unroll
         for (int np = 0; np < DV / 16; ++np) {
           uint32_t b0, b1, b2, b3;  // (d_v n-tile 2np: queries lo, hi), (2np+1: lo, hi)
@@ -274,9 +281,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
           mma16816(dv_acc[2 * np + 1], pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3], b2, b3);
         }
       }
-      // ---- dK += dS^T Q (16 keys x r), k = 32 queries (scale applied at the end)
+      // ---- dK += dS^T Q (16 keys x r), k = kPartQ queries (scale applied at the end)
 #pragma unroll
-      for (int kk = 0; kk < 2; ++kk) {
+      for (int kk = 0; kk < kPartQ / 16; ++kk) {
 #pragma unroll
         for (int np = 0; np < R / 16; ++np) {
           uint32_t b0, b1, b2, b3;
@@ -285,9 +292,11 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
           mma16816(dk_acc[2 * np + 1], da[kk][0], da[kk][1], da[kk][2], da[kk][3], b2, b3);
         }
       }
-      // ---- dQ += dS K (32 queries x r), k = this warp's 16 keys: dS via movmatrix
+      // ---- dQ += dS K (kPartQ queries x r), k = this warp's 16 keys: dS via movmatrix;
+      // the warp's partial goes to its own buffer, the four are summed below
+      float* mine = dqw + warp * kPartQ * C::DQP;
 #pragma unroll
-      for (int mt = 0; mt < 2; ++mt) {
+      for (int mt = 0; mt < kPartQ / 16; ++mt) {
         const uint32_t a0 = movm_t(da[mt][0]);   // queries 16mt+g8,   keys 2t4..   (key block 0-7)
         const uint32_t a1 = movm_t(da[mt][2]);   // queries 16mt+8+g8, keys 2t4..
         const uint32_t a2 = movm_t(da[mt][1]);   // queries 16mt+g8,   keys 8+2t4..
@@ -299,30 +308,35 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
           float c0[4] = {0.f, 0.f, 0.f, 0.f}, c1[4] = {0.f, 0.f, 0.f, 0.f};
           mma16816(c0, a0, a1, a2, a3, b0, b1);
           mma16816(c1, a0, a1, a2, a3, b2, b3);
-          const int q0 = qb + 16 * mt + g8;
+          const int q0 = 16 * mt + g8;            // query within the half
           const int r0 = 16 * np + 2 * t4;
-          atomicAdd(&dqacc[q0 * R + r0], c0[0]);
-          atomicAdd(&dqacc[q0 * R + r0 + 1], c0[1]);
-          atomicAdd(&dqacc[(q0 + 8) * R + r0], c0[2]);
-          atomicAdd(&dqacc[(q0 + 8) * R + r0 + 1], c0[3]);
-          atomicAdd(&dqacc[q0 * R + r0 + 8], c1[0]);
-          atomicAdd(&dqacc[q0 * R + r0 + 9], c1[1]);
-          atomicAdd(&dqacc[(q0 + 8) * R + r0 + 8], c1[2]);
-          atomicAdd(&dqacc[(q0 + 8) * R + r0 + 9], c1[3]);
+          *reinterpret_cast<float2*>(mine + q0 * C::DQP + r0) = make_float2(c0[0], c0[1]);
+          *reinterpret_cast<float2*>(mine + (q0 + 8) * C::DQP + r0) = make_float2(c0[2], c0[3]);
+          *reinterpret_cast<float2*>(mine + q0 * C::DQP + r0 + 8) = make_float2(c1[0], c1[1]);
+          *reinterpret_cast<float2*>(mine + (q0 + 8) * C::DQP + r0 + 8) = make_float2(c1[2], c1[3]);
         }
       }
-    }
-    __syncthreads();
-    // this CTA's dQ contribution for query tile i of head h
-    {
-      const int rows = min(kTile, S - i * kTile);
-      float* dq = p.dq + ((static_cast<size_t>(b) * p.Hq + h) * S + static_cast<size_t>(i) * kTile) * R;
-      for (int e = tid; e < kTile * R; e += kBwdThreads) {
-        if (e / R < rows) atomicAdd(&dq[e], dqacc[e] * p.scale);
-        dqacc[e] = 0.f;
+      __syncthreads();
+      // the part's dQ: the four warps' partials summed, added into dq (4 floats at a time)
+      {
+        const int rows = min(kPartQ, S - i * kTile - qb);
+        float* dq = p.dq + ((static_cast<size_t>(b) * p.Hq + h) * S + static_cast<size_t>(i) * kTile + qb) * R;
+#pragma unroll 1
+        for (int e = tid * 4; e < kPartQ * R; e += kBwdThreads * 4) {
+          const int q = e / R, c = e % R;
+          if (q >= rows) continue;
+          float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            const float4 x = *reinterpret_cast<const float4*>(dqw + (w * kPartQ + q) * C::DQP + c);
+            sum.x += x.x; sum.y += x.y; sum.z += x.z; sum.w += x.w;
+          }
+          sum.x *= p.scale; sum.y *= p.scale; sum.z *= p.scale; sum.w *= p.scale;
+          atomicAdd(reinterpret_cast<float4*>(dq + e), sum);
+        }
       }
+      __syncthreads();
     }
-    __syncthreads();
   }
   cp_async_wait<0>();
 
