@@ -17,7 +17,8 @@
 //         S^T = K Q^T and P^T = exp2(S^T scale log2e - lse log2e)   (recomputed)
 //         dP^T = V dO^T,  dS^T = P^T * (dP^T - D)
 //         dV += P^T dO,   dK += dS^T Q                     (registers, whole run)
-//         dQ(i) += dS K   (warps summed in shared memory, CTAs with fp32 atomics)
+//         dQ(i) += dS K   (per-warp partials in shared memory, summed and added
+//                          to global dQ with float4 atomics, once per query part)
 //     P^T and dS^T go from the accumulator layout straight into the A operand
 //     of the next products; dS is transposed for dQ with movmatrix.  Q, dO and
 //     the per-row statistics stream through a double-buffered cp.async ring
@@ -33,11 +34,6 @@ namespace {
 
 constexpr int kTile = 64;       // keys per CTA, queries per visit
 constexpr int kBwdThreads = 128;
-#ifndef TK_BWD_PARTQ
-#define TK_BWD_PARTQ 16
-#endif
-constexpr int kPartQ = TK_BWD_PARTQ;   // queries per step of a visit (fragments held at once)
-constexpr int kParts = kTile / kPartQ;
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& a, uint32_t& b, uint32_t& c,
                                         uint32_t& d) {
@@ -133,6 +129,9 @@ __global__ void __launch_bounds__(256) bwd_prep(const BackwardParams p) {
 template <int R, int DV>
 struct BCfg {
   static constexpr int KW = R * 2, VW = DV * 2;   // bytes per K / Q row and V / dO row
+  // queries per step of a visit: the S^T / dP^T fragments of a step are held at once
+  // (32 fits in registers up to r = 64; at r = 128 the dK / dQ fragments leave room for 16)
+  static constexpr int PQ = R <= 64 ? 32 : 16, PARTS = kTile / PQ;
   static constexpr int OFF_K = 0;
   static constexpr int OFF_V = OFF_K + kTile * KW;
   static constexpr int OFF_BUF = OFF_V + kTile * VW;
@@ -141,8 +140,8 @@ struct BCfg {
   // dQ partials of one part of the queries, one buffer per warp, rows padded to R + 8
   // floats so that a warp's 64-bit fragment stores hit 32 different banks
   static constexpr int DQP = R + 8;
-  static constexpr int OFF_DQ = OFF_BUF + 2 * BUF;          // [4 warps][kPartQ][DQP] fp32
-  static constexpr int SMEM = OFF_DQ + 4 * kPartQ * DQP * 4;
+  static constexpr int OFF_DQ = OFF_BUF + 2 * BUF;          // [4 warps][PQ][DQP] fp32
+  static constexpr int SMEM = OFF_DQ + 4 * PQ * DQP * 4;
   static_assert(SMEM <= 227 * 1024, "shared memory");
 };
 
@@ -213,31 +212,31 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
     const bool diag = p.causal && i == j;
 
 #pragma unroll 1
-    for (int part = 0; part < kParts; ++part) {
-      const int qb = part * kPartQ;                 // first query (in the tile) of this part
-      float sa[kPartQ / 8][4], dp[kPartQ / 8][4];
+    for (int part = 0; part < C::PARTS; ++part) {
+      const int qb = part * C::PQ;                 // first query (in the tile) of this part
+      float sa[C::PQ / 8][4], dp[C::PQ / 8][4];
 #pragma unroll
-      for (int n = 0; n < kPartQ / 8; ++n) sa[n][0] = sa[n][1] = sa[n][2] = sa[n][3] = dp[n][0] = dp[n][1] = dp[n][2] = dp[n][3] = 0.f;
-      // ---- S^T = K Q^T (16 keys x kPartQ queries), k = r
+      for (int n = 0; n < C::PQ / 8; ++n) sa[n][0] = sa[n][1] = sa[n][2] = sa[n][3] = dp[n][0] = dp[n][1] = dp[n][2] = dp[n][3] = 0.f;
+      // ---- S^T = K Q^T (16 keys x PQ queries), k = r
 #pragma unroll
       for (int ks = 0; ks < R / 16; ++ks) {
         uint32_t a0, a1, a2, a3;
         ldsm_x4(sbase + C::OFF_K + swz<C::KW>(krow + (mi & 1) * 8 + rr, 2 * ks + (mi >> 1)), a0, a1, a2, a3);
 #pragma unroll
-        for (int np = 0; np < kPartQ / 16; ++np) {
+        for (int np = 0; np < C::PQ / 16; ++np) {
           uint32_t b0, b1, b2, b3;  // queries qb+16np.. : (n-tile 2np, k lo/hi), (2np+1, k lo/hi)
           ldsm_x4(bq + swz<C::KW>(qb + 16 * np + (mi >> 1) * 8 + rr, 2 * ks + (mi & 1)), b0, b1, b2, b3);
           mma16816(sa[2 * np], a0, a1, a2, a3, b0, b1);
           mma16816(sa[2 * np + 1], a0, a1, a2, a3, b2, b3);
         }
       }
-      // ---- dP^T = V dO^T (16 keys x kPartQ queries), k = d_v
+      // ---- dP^T = V dO^T (16 keys x PQ queries), k = d_v
 #pragma unroll
       for (int ks = 0; ks < DV / 16; ++ks) {
         uint32_t a0, a1, a2, a3;
         ldsm_x4(sbase + C::OFF_V + swz<C::VW>(krow + (mi & 1) * 8 + rr, 2 * ks + (mi >> 1)), a0, a1, a2, a3);
 #pragma unroll
-        for (int np = 0; np < kPartQ / 16; ++np) {
+        for (int np = 0; np < C::PQ / 16; ++np) {
           uint32_t b0, b1, b2, b3;
           ldsm_x4(bdo + swz<C::VW>(qb + 16 * np + (mi >> 1) * 8 + rr, 2 * ks + (mi & 1)), b0, b1, b2, b3);
           mma16816(dp[2 * np], a0, a1, a2, a3, b0, b1);
@@ -246,7 +245,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
       }
       // ---- P^T and dS^T in the accumulator layout: (key g8 | g8+8, query 2t4 | 2t4+1)
 #pragma unroll
-      for (int n = 0; n < kPartQ / 8; ++n) {
+      for (int n = 0; n < C::PQ / 8; ++n) {
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const int q = qb + 8 * n + 2 * t4 + (e & 1);     // query in the tile
@@ -257,10 +256,10 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
           dp[n][e] = pr * (dp[n][e] - dsum[q]);
         }
       }
-      // A operands (16 keys x 16 queries) of P^T and dS^T for the two 16-query steps
-      uint32_t pa[kPartQ / 16][4], da[kPartQ / 16][4];
+      // A operands (16 keys x 16 queries) of P^T and dS^T for each 16-query k-step
+      uint32_t pa[C::PQ / 16][4], da[C::PQ / 16][4];
 #pragma unroll
-      for (int kk = 0; kk < kPartQ / 16; ++kk) {
+      for (int kk = 0; kk < C::PQ / 16; ++kk) {
         pa[kk][0] = pack_bf16(sa[2 * kk][0], sa[2 * kk][1]);
         pa[kk][1] = pack_bf16(sa[2 * kk][2], sa[2 * kk][3]);
         pa[kk][2] = pack_bf16(sa[2 * kk + 1][0], sa[2 * kk + 1][1]);
@@ -270,9 +269,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
         da[kk][2] = pack_bf16(dp[2 * kk + 1][0], dp[2 * kk + 1][1]);
         da[kk][3] = pack_bf16(dp[2 * kk + 1][2], dp[2 * kk + 1][3]);
       }
-      // ---- dV += P^T dO (16 keys x d_v), k = kPartQ queries
+      // ---- dV += P^T dO (16 keys x d_v), k = PQ queries
 #pragma unroll
-      for (int kk = 0; kk < kPartQ / 16; ++kk) {
+      for (int kk = 0; kk < C::PQ / 16; ++kk) {
 #pragma unroll
         for (int np = 0; np < DV / 16; ++np) {
           uint32_t b0, b1, b2, b3;  // (d_v n-tile 2np: queries lo, hi), (2np+1: lo, hi)
@@ -281,9 +280,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
           mma16816(dv_acc[2 * np + 1], pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3], b2, b3);
         }
       }
-      // ---- dK += dS^T Q (16 keys x r), k = kPartQ queries (scale applied at the end)
+      // ---- dK += dS^T Q (16 keys x r), k = PQ queries (scale applied at the end)
 #pragma unroll
-      for (int kk = 0; kk < kPartQ / 16; ++kk) {
+      for (int kk = 0; kk < C::PQ / 16; ++kk) {
 #pragma unroll
         for (int np = 0; np < R / 16; ++np) {
           uint32_t b0, b1, b2, b3;
@@ -292,11 +291,11 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
           mma16816(dk_acc[2 * np + 1], da[kk][0], da[kk][1], da[kk][2], da[kk][3], b2, b3);
         }
       }
-      // ---- dQ += dS K (kPartQ queries x r), k = this warp's 16 keys: dS via movmatrix;
+      // ---- dQ += dS K (PQ queries x r), k = this warp's 16 keys: dS via movmatrix;
       // the warp's partial goes to its own buffer, the four are summed below
-      float* mine = dqw + warp * kPartQ * C::DQP;
+      float* mine = dqw + warp * C::PQ * C::DQP;
 #pragma unroll
-      for (int mt = 0; mt < kPartQ / 16; ++mt) {
+      for (int mt = 0; mt < C::PQ / 16; ++mt) {
         const uint32_t a0 = movm_t(da[mt][0]);   // queries 16mt+g8,   keys 2t4..   (key block 0-7)
         const uint32_t a1 = movm_t(da[mt][2]);   // queries 16mt+8+g8, keys 2t4..
         const uint32_t a2 = movm_t(da[mt][1]);   // queries 16mt+g8,   keys 8+2t4..
@@ -319,16 +318,16 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
       __syncthreads();
       // the part's dQ: the four warps' partials summed, added into dq (4 floats at a time)
       {
-        const int rows = min(kPartQ, S - i * kTile - qb);
+        const int rows = min(C::PQ, S - i * kTile - qb);
         float* dq = p.dq + ((static_cast<size_t>(b) * p.Hq + h) * S + static_cast<size_t>(i) * kTile + qb) * R;
 #pragma unroll 1
-        for (int e = tid * 4; e < kPartQ * R; e += kBwdThreads * 4) {
+        for (int e = tid * 4; e < C::PQ * R; e += kBwdThreads * 4) {
           const int q = e / R, c = e % R;
           if (q >= rows) continue;
           float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
           for (int w = 0; w < 4; ++w) {
-            const float4 x = *reinterpret_cast<const float4*>(dqw + (w * kPartQ + q) * C::DQP + c);
+            const float4 x = *reinterpret_cast<const float4*>(dqw + (w * C::PQ + q) * C::DQP + c);
             sum.x += x.x; sum.y += x.y; sum.z += x.z; sum.w += x.w;
           }
           sum.x *= p.scale; sum.y *= p.scale; sum.z *= p.scale; sum.w *= p.scale;
