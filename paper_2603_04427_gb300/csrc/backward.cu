@@ -9,12 +9,16 @@
 // (D_i equals rowsum(dP * p) for the exact forward output).
 //
 // Two kernels:
-//   bwd_prep: D = rowsum(dO * out) per query row, and dQ set to zero.
+//   bwd_prep: D = rowsum(dO * out) and lse2 = lse log2(e) per query row (rows
+//     padded to a multiple of 128), and dQ set to zero.
+//   the gradient kernel: for r <= 64 the tensor-memory kernel of
+//     backward_tc.cu; for r = 128 (whose TMEM accumulators do not fit beside
+//     the score tiles) bwd_main below.
 //   bwd_main: one CTA per (sequence, kv head g, 64-key tile j); 4 warps, warp
 //     w owns keys 16w..16w+15 of the tile.  It visits every query tile i (64
 //     rows; i >= j when causal) of each of the G query heads of g and, on the
 //     tensor cores with mma.sync.m16n8k16 (bf16 operands, fp32 accumulation):
-//         S^T = K Q^T and P^T = exp2(S^T scale log2e - lse log2e)   (recomputed)
+//         S^T = K Q^T and P^T = exp2(S^T scale log2e - lse2)   (recomputed)
 //         dP^T = V dO^T,  dS^T = P^T * (dP^T - D)
 //         dV += P^T dO,   dK += dS^T Q                     (registers, whole run)
 //         dQ(i) += dS K   (per-warp partials in shared memory, summed and added
@@ -106,23 +110,38 @@ __device__ __forceinline__ void load_tile(uint32_t dst, const unsigned char* src
 }
 
 // ---------------------------------------------------------------- preprocessing
-// One warp per query row: D = sum_c dO * out (fp32), and the row of dQ zeroed.
+// One warp per padded statistics row (b, h, i < S_pad): for i < S,
+// D = sum_c dO * out (fp32), lse2 = lse * log2(e) and the row of dQ zeroed;
+// for S <= i < S_pad, D = 0 and lse2 = +inf (such rows get softmax weight 0).
 template <int R, int DV>
 __global__ void __launch_bounds__(256) bwd_prep(const BackwardParams p) {
   const long long row = static_cast<long long>(blockIdx.x) * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
-  const long long rows = static_cast<long long>(p.B) * p.Hq * p.S;
+  const long long rows = static_cast<long long>(p.B) * p.Hq * p.S_pad;
   if (row >= rows) return;
-  const __nv_bfloat16* o = static_cast<const __nv_bfloat16*>(p.out) + row * DV;
-  const __nv_bfloat16* d = static_cast<const __nv_bfloat16*>(p.d_out) + row * DV;
+  const long long bh = row / p.S_pad;
+  const int i = static_cast<int>(row - bh * p.S_pad);
+  if (i >= p.S) {
+    if (lane == 0) {
+      p.dsum[row] = 0.f;
+      p.lse2[row] = INFINITY;
+    }
+    return;
+  }
+  const long long x = bh * p.S + i;   // row of the [B][Hq][S] tensors
+  const __nv_bfloat16* o = static_cast<const __nv_bfloat16*>(p.out) + x * DV;
+  const __nv_bfloat16* d = static_cast<const __nv_bfloat16*>(p.d_out) + x * DV;
   float acc = 0.f;
 #pragma unroll
   for (int c = lane; c < DV; c += 32) acc += __bfloat162float(o[c]) * __bfloat162float(d[c]);
 #pragma unroll
   for (int off = 16; off >= 1; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-  if (lane == 0) p.dsum[row] = acc;
+  if (lane == 0) {
+    p.dsum[row] = acc;
+    p.lse2[row] = p.lse[x] * 1.4426950408889634f;
+  }
 #pragma unroll
-  for (int c = lane; c < R; c += 32) p.dq[row * R + c] = 0.f;
+  for (int c = lane; c < R; c += 32) p.dq[x * R + c] = 0.f;
 }
 
 // ---------------------------------------------------------------- main kernel
@@ -180,11 +199,10 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
     const uint32_t bb = sbase + C::OFF_BUF + buf * C::BUF;
     load_tile<C::KW>(bb + C::BUF_Q, static_cast<const unsigned char*>(p.q) + qrow * C::KW, rows, tid);
     load_tile<C::VW>(bb + C::BUF_DO, static_cast<const unsigned char*>(p.d_out) + qrow * C::VW, rows, tid);
-    {  // the rows' statistics: threads 0-63 the logsumexp, 64-127 D (4 bytes each)
+    {  // the rows' statistics (padded rows: always in range): threads 0-63 lse2, 64-127 D
       const int r = tid & (kTile - 1);
-      const bool valid = r < rows;
-      cp_async4(bb + (tid < kTile ? C::BUF_LSE : C::BUF_D) + r * 4,
-                (tid < kTile ? p.lse : p.dsum) + qrow + (valid ? r : 0), valid);
+      const size_t srow = (static_cast<size_t>(b) * p.Hq + h) * p.S_pad + static_cast<size_t>(i) * kTile + r;
+      cp_async4(bb + (tid < kTile ? C::BUF_LSE : C::BUF_D) + r * 4, (tid < kTile ? p.lse2 : p.dsum) + srow, true);
     }
   };
   if (visits > 0) load_visit(0, 0);
@@ -207,7 +225,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
     const int h = g * G + vis / per_head, i = i0 + vis % per_head;
     const uint32_t bq = sbase + C::OFF_BUF + cur * C::BUF + C::BUF_Q;
     const uint32_t bdo = sbase + C::OFF_BUF + cur * C::BUF + C::BUF_DO;
-    const float* lse = reinterpret_cast<const float*>(smem + C::OFF_BUF + cur * C::BUF + C::BUF_LSE);
+    const float* lse2 = reinterpret_cast<const float*>(smem + C::OFF_BUF + cur * C::BUF + C::BUF_LSE);
     const float* dsum = reinterpret_cast<const float*>(smem + C::OFF_BUF + cur * C::BUF + C::BUF_D);
     const bool diag = p.causal && i == j;
 
@@ -251,7 +269,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
           const int q = qb + 8 * n + 2 * t4 + (e & 1);     // query in the tile
           const int key = key0 + (e >> 1) * 8;              // absolute key
           const bool hide = diag && key > i * kTile + q;
-          const float pr = hide ? 0.f : fast_exp2(sa[n][e] * sl2 - lse[q] * 1.4426950408889634f);
+          const float pr = hide ? 0.f : fast_exp2(sa[n][e] * sl2 - lse2[q]);
           sa[n][e] = pr;
           dp[n][e] = pr * (dp[n][e] - dsum[q]);
         }
@@ -358,28 +376,32 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
 }
 
 template <int R, int DV>
-cudaError_t launch_t(const BackwardParams& p, cudaStream_t s) {
-  using C = BCfg<R, DV>;
-  const long long rows = static_cast<long long>(p.B) * p.Hq * p.S;
+cudaError_t launch_t(const BackwardParams& p, cudaStream_t s, int* uns) {
+  const long long rows = static_cast<long long>(p.B) * p.Hq * p.S_pad;
   const long long pblocks = (rows + 7) / 8;
   if (pblocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
   bwd_prep<R, DV><<<static_cast<unsigned>(pblocks), 256, 0, s>>>(p);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(bwd_main<R, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-  if (e != cudaSuccess) return e;
-  const long long n_t = (p.S + kTile - 1) / kTile;
-  const long long grid = static_cast<long long>(p.B) * p.Hkv * n_t;
-  if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-  bwd_main<R, DV><<<static_cast<unsigned>(grid), kBwdThreads, C::SMEM, s>>>(p);
-  return cudaGetLastError();
+  if constexpr (R <= 64) {
+    return launch_backward_tc(p, s, uns);
+  } else {
+    using C = BCfg<R, DV>;
+    e = cudaFuncSetAttribute(bwd_main<R, DV>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    if (e != cudaSuccess) return e;
+    const long long n_t = (p.S + kTile - 1) / kTile;
+    const long long grid = static_cast<long long>(p.B) * p.Hkv * n_t;
+    if (grid > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    bwd_main<R, DV><<<static_cast<unsigned>(grid), kBwdThreads, C::SMEM, s>>>(p);
+    return cudaGetLastError();
+  }
 }
 
 template <int R>
 cudaError_t by_dv(const BackwardParams& p, cudaStream_t s, int* uns) {
   switch (p.DV) {
-    case 64: return launch_t<R, 64>(p, s);
-    case 128: return launch_t<R, 128>(p, s);
+    case 64: return launch_t<R, 64>(p, s, uns);
+    case 128: return launch_t<R, 128>(p, s, uns);
   }
   *uns = 1;
   return cudaSuccess;

@@ -113,13 +113,21 @@ struct BackwardParams {
   float* dq;          // fp32 [B][Hq][S][R]  (accumulated: zeroed by the preprocessing kernel)
   float* dk;          // fp32 [B][Hkv][S][R]
   float* dv;          // fp32 [B][Hkv][S][DV]
-  float* dsum;        // [B][Hq][S] workspace: rowsum(d_out * out)
-  int B, Hq, Hkv, S, R, DV;
+  // workspace, rows padded to S_pad (a multiple of 128) per (b, query head):
+  float* lse2;        // [B*Hq][S_pad] lse * log2(e); +inf on rows >= S (weight 0)
+  float* dsum;        // [B*Hq][S_pad] rowsum(d_out * out); 0 on rows >= S
+  int* err;
+  int B, Hq, Hkv, S, S_pad, R, DV;
   int causal;
   float scale;
 };
 
+// Rows of the backward's per-row statistics: S rounded up to 128.
+inline int backward_rows(int S) { return (S + 127) / 128 * 128; }
+
 cudaError_t launch_backward(const BackwardParams& p, cudaStream_t stream, int* unsupported);
+// The tensor-memory gradient kernel (r <= 64), after the preprocessing pass.
+cudaError_t launch_backward_tc(const BackwardParams& p, cudaStream_t stream, int* unsupported);
 
 cudaError_t launch_prefill(const PrefillParams& p, cudaStream_t stream, int* unsupported);
 

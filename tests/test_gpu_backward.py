@@ -54,7 +54,7 @@ def _case(B, hq, hkv, S, r, dv, causal, seed):
 
 
 @pytest.mark.parametrize("causal", [True, False])
-@pytest.mark.parametrize("r,dv", [(32, 128), (16, 64), (64, 128), (128, 64)])
+@pytest.mark.parametrize("r,dv", [(32, 128), (16, 64), (64, 128), (128, 64), (16, 128), (32, 64), (64, 64), (128, 128)])
 def test_backward_matches_oracle(r, dv, causal):
     require_gpu()
     B, hq, hkv, S = 2, 4, 2, 300
@@ -89,3 +89,14 @@ def test_backward_7b_shape_sampled_heads():
         _grad_parity(f64(dq[:, sl]), rq, f"7b dq head {h}")
         _grad_parity(f64(dk[:, sl]), rk, f"7b dk head {h}")
         _grad_parity(f64(dvv[:, sl]), rv, f"7b dv head {h}")
+
+
+@pytest.mark.parametrize("r", [16, 32, 64])
+def test_backward_gqa_many_tiles(r):
+    """G = 8 query heads per kv head, several key and query tiles and a ragged tail."""
+    require_gpu()
+    B, hq, hkv, S, dv = 1, 16, 2, 777, 128
+    q, k, v, do, lse, dq, dk, dvv = _case(B, hq, hkv, S, r, dv, True, seed=70 + r)
+    rq, rk, rv = oa.attention_backward(f64(q), f64(k), f64(v), f64(do), 1 / math.sqrt(r))
+    for got, ref, n in ((dq, rq, "dq"), (dk, rk, "dk"), (dvv, rv, "dv")):
+        _grad_parity(f64(got), ref, f"{n} G=8 r={r}")
