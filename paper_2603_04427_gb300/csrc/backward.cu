@@ -9,7 +9,7 @@
 // (D_i equals rowsum(dP * p) for the exact forward output).
 //
 // Two kernels:
-//   bwd_prep: D = rowsum(dO * out) and lse2 = lse log2(e) per query row (rows
+//   bwd_prep: -D = -rowsum(dO * out) and -lse log2(e) per query row (rows
 //     padded to a multiple of 128), and dQ set to zero.
 //   the gradient kernel: for r <= 64 the tensor-memory kernel of
 //     backward_tc.cu; for r = 128 (whose TMEM accumulators do not fit beside
@@ -18,7 +18,7 @@
 //     w owns keys 16w..16w+15 of the tile.  It visits every query tile i (64
 //     rows; i >= j when causal) of each of the G query heads of g and, on the
 //     tensor cores with mma.sync.m16n8k16 (bf16 operands, fp32 accumulation):
-//         S^T = K Q^T and P^T = exp2(S^T scale log2e - lse2)   (recomputed)
+//         S^T = K Q^T and P^T = exp2(S^T scale log2e - lse log2e)   (recomputed)
 //         dP^T = V dO^T,  dS^T = P^T * (dP^T - D)
 //         dV += P^T dO,   dK += dS^T Q                     (registers, whole run)
 //         dQ(i) += dS K   (per-warp partials in shared memory, summed and added
@@ -111,8 +111,8 @@ __device__ __forceinline__ void load_tile(uint32_t dst, const unsigned char* src
 
 // ---------------------------------------------------------------- preprocessing
 // One warp per padded statistics row (b, h, i < S_pad): for i < S,
-// D = sum_c dO * out (fp32), lse2 = lse * log2(e) and the row of dQ zeroed;
-// for S <= i < S_pad, D = 0 and lse2 = +inf (such rows get softmax weight 0).
+// nd = -sum_c dO * out (fp32), nl2 = -lse * log2(e) and the row of dQ zeroed;
+// for S <= i < S_pad, nd = 0 and nl2 = -inf (such rows get softmax weight 0).
 template <int R, int DV>
 __global__ void __launch_bounds__(256) bwd_prep(const BackwardParams p) {
   const long long row = static_cast<long long>(blockIdx.x) * 8 + (threadIdx.x >> 5);
@@ -123,8 +123,8 @@ __global__ void __launch_bounds__(256) bwd_prep(const BackwardParams p) {
   const int i = static_cast<int>(row - bh * p.S_pad);
   if (i >= p.S) {
     if (lane == 0) {
-      p.dsum[row] = 0.f;
-      p.lse2[row] = INFINITY;
+      p.nd[row] = 0.f;
+      p.nl2[row] = -INFINITY;
     }
     return;
   }
@@ -137,8 +137,8 @@ __global__ void __launch_bounds__(256) bwd_prep(const BackwardParams p) {
 #pragma unroll
   for (int off = 16; off >= 1; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
   if (lane == 0) {
-    p.dsum[row] = acc;
-    p.lse2[row] = p.lse[x] * 1.4426950408889634f;
+    p.nd[row] = -acc;
+    p.nl2[row] = -p.lse[x] * 1.4426950408889634f;
   }
 #pragma unroll
   for (int c = lane; c < R; c += 32) p.dq[x * R + c] = 0.f;
@@ -199,10 +199,10 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
     const uint32_t bb = sbase + C::OFF_BUF + buf * C::BUF;
     load_tile<C::KW>(bb + C::BUF_Q, static_cast<const unsigned char*>(p.q) + qrow * C::KW, rows, tid);
     load_tile<C::VW>(bb + C::BUF_DO, static_cast<const unsigned char*>(p.d_out) + qrow * C::VW, rows, tid);
-    {  // the rows' statistics (padded rows: always in range): threads 0-63 lse2, 64-127 D
+    {  // the rows' statistics (padded rows: always in range): threads 0-63 nl2, 64-127 nd
       const int r = tid & (kTile - 1);
       const size_t srow = (static_cast<size_t>(b) * p.Hq + h) * p.S_pad + static_cast<size_t>(i) * kTile + r;
-      cp_async4(bb + (tid < kTile ? C::BUF_LSE : C::BUF_D) + r * 4, (tid < kTile ? p.lse2 : p.dsum) + srow, true);
+      cp_async4(bb + (tid < kTile ? C::BUF_LSE : C::BUF_D) + r * 4, (tid < kTile ? p.nl2 : p.nd) + srow, true);
     }
   };
   if (visits > 0) load_visit(0, 0);
@@ -225,8 +225,8 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
     const int h = g * G + vis / per_head, i = i0 + vis % per_head;
     const uint32_t bq = sbase + C::OFF_BUF + cur * C::BUF + C::BUF_Q;
     const uint32_t bdo = sbase + C::OFF_BUF + cur * C::BUF + C::BUF_DO;
-    const float* lse2 = reinterpret_cast<const float*>(smem + C::OFF_BUF + cur * C::BUF + C::BUF_LSE);
-    const float* dsum = reinterpret_cast<const float*>(smem + C::OFF_BUF + cur * C::BUF + C::BUF_D);
+    const float* nl2 = reinterpret_cast<const float*>(smem + C::OFF_BUF + cur * C::BUF + C::BUF_LSE);
+    const float* nd = reinterpret_cast<const float*>(smem + C::OFF_BUF + cur * C::BUF + C::BUF_D);
     const bool diag = p.causal && i == j;
 
 #pragma unroll 1
@@ -269,9 +269,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
           const int q = qb + 8 * n + 2 * t4 + (e & 1);     // query in the tile
           const int key = key0 + (e >> 1) * 8;              // absolute key
           const bool hide = diag && key > i * kTile + q;
-          const float pr = hide ? 0.f : fast_exp2(sa[n][e] * sl2 - lse2[q]);
+          const float pr = hide ? 0.f : fast_exp2(fmaf(sa[n][e], sl2, nl2[q]));
           sa[n][e] = pr;
-          dp[n][e] = pr * (dp[n][e] - dsum[q]);
+          dp[n][e] = pr * (dp[n][e] + nd[q]);
         }
       }
       // A operands (16 keys x 16 queries) of P^T and dS^T for each 16-query k-step

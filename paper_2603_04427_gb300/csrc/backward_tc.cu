@@ -7,37 +7,42 @@
 // (masked) and dL/d(out) = dO:
 //     dV = p^T dO,  dP = dO v^T,  dS = p * (dP - D),  D_i = sum_c dO_ic out_ic,
 //     dQ = scale dS k,  dK = scale dS^T q.
-// The preprocessing pass (backward.cu) has written D and lse2 = lse log2(e)
-// for every query row, padded to a multiple of 128 rows (lse2 = +inf, D = 0 on
-// the padding), and zeroed dQ.
+// The preprocessing pass (backward.cu) has written -lse log2(e) and -D for
+// every query row, padded to a multiple of 128 rows (-inf and 0 on the
+// padding: such rows get weight 0), and zeroed dQ.
 //
 // One CTA per (sequence, kv head g, 128-key tile j).  Keys are the MMA's M
 // dimension and the TMEM lanes: thread t of a 4-warp group owns key t.  The
 // CTA visits every 128-query tile i (i >= j when causal) of each of the G
 // query heads of g, as two 64-query halves h:
-//   warp 12 (one lane): TMA loads of K_j, V_j (once) and, per tile, of Q_i,
-//       dO_i and the rows' lse2 / D into a 2-stage ring.
-//   warp 13 (whole warp, one elected lane issues): per tile and half
+//   warp 9 (one lane): TMA loads of K_j, V_j (once) and, per half tile, of
+//       Q, dO and the rows' statistics into a 4-slot ring.
+//   warp 8 (whole warp, one elected lane issues): per tile and half
 //       S^T_h  = K Q_h^T     (M=128 keys, N=64 queries, K=r)
 //       dP^T_h = V dO_h^T    (M=128, N=64, K=d_v)
 //       dV    += P^T_h dO_h  (N=d_v, K=64; P^T_h read from TMEM)
 //       dK    += dS^T_h Q_h  (N=r,   K=64; dS^T_h from shared memory, K-major)
 //     and per tile  dQ_i = dS K  (M=128 queries, N=r, K=128 keys; dS from the
 //     same shared-memory tile read MN-major), completion on mbarriers through
-//     tcgen05.commit.  The next tile's S / dP products of a half are issued as
-//     soon as that half's P has been consumed, so one half's softmax overlaps
-//     the other half's products.
+//     tcgen05.commit.  Where TMEM has room for P^T in columns of its own and
+//     shared memory for two dS tiles (the EARLY schedule), the next tile's
+//     S / dP products of a half are issued as soon as the half's softmax warps
+//     have read S / dP into registers, and a tile's dQ product during the next
+//     tile; otherwise each half's products follow its softmax.
 //   warps 0-3 / 4-7 (half 0 / 1): read S^T_h and dP^T_h from TMEM, form
-//       P^T = exp2(S^T scale log2e - lse2) (masked) and dS^T = P^T (dP^T - D),
-//       write P^T as bf16 into TMEM over S^T_h and dS^T as bf16 into the
-//       swizzled shared-memory tile.
-//   warps 8-11 (thread t owns query t of the tile): read dQ_i from TMEM and
-//       add it into global dq with one bulk reduce-add per row
-//       (cp.reduce.async.bulk .add.f32); at the end, dK (times scale) and dV
-//       of the CTA's keys from TMEM to global memory.
+//       P^T = exp2(S^T scale log2e - lse log2e) (masked) and
+//       dS^T = P^T (dP^T - D) in packed fp32 pairs, write P^T as bf16 into
+//       TMEM and dS^T as bf16 into the swizzled shared-memory tile.  Then each
+//       warpgroup adds half of the previous tile's dQ columns (thread t: query
+//       t) into global dq: staged in shared memory, one TMA tensor reduce-add
+//       (cp.reduce.async.bulk.tensor .add) per warp.  At the end warps 0-3
+//       store dK (times scale) and the first half of dV's columns, warps 4-7
+//       the second half.
+// 10 warps, so that a thread may hold 168 registers.
 //
-// TMEM columns: [0,64) S^T_0 (P^T_0 in its first 32), [64,128) dP^T_0,
-// [128,192) S^T_1, [192,256) dP^T_1, then dV (d_v), dK (r), dQ (r).
+// TMEM columns: [0,64) S^T_0, [64,128) dP^T_0, [128,192) S^T_1,
+// [192,256) dP^T_1, then dV (d_v), dK (r), dQ (r), and where they fit P^T_0,
+// P^T_1 (32 columns each; otherwise P^T_h sits in the first 32 of S^T_h).
 #include <algorithm>
 #include <type_traits>
 
@@ -51,7 +56,7 @@ namespace {
 constexpr int kKeys = 128;         // keys per CTA (MMA M, TMEM lanes)
 constexpr int kQT = 128;           // queries per tile
 constexpr int kHalfQ = 64;         // queries per S / dP half
-constexpr int kTcThreads = 448;    // 3 x 4 warps, the TMA warp, the MMA warp
+constexpr int kTcThreads = 320;    // 2 x 4 softmax warps, the MMA warp, the TMA warp
 constexpr int kTmemColsTc = 512;
 constexpr int kBoxB = 128 * 128;   // one 64-column (128-byte) box of a 128-row tile
 
@@ -65,31 +70,47 @@ struct TCfg {
   static constexpr uint32_t QK_LAYOUT = QK_SW == 32 ? 6u : (QK_SW == 64 ? 4u : 2u);
   static constexpr int KB = kKeys * R * 2;         // K tile
   static constexpr int VB = kKeys * DV * 2;        // V tile (DV / 64 boxes)
-  static constexpr int QB = kQT * R * 2;           // Q tile
-  static constexpr int OB = kQT * DV * 2;          // dO tile (DV / 64 boxes)
-  static constexpr int ST_Q = 0, ST_O = align1k(QB), ST_LSE = ST_O + OB, ST_D = ST_LSE + kQT * 4;
-  static constexpr int STAGE = ST_D + kQT * 4;      // multiple of 1024
+  // Q / dO arrive in 64-query half tiles, a ring of 4 slots: a slot is
+  // released as soon as its half's dV / dK products have read it
+  static constexpr int QHB = kHalfQ * R * 2;       // Q half tile (one box)
+  static constexpr int OHB = kHalfQ * DV * 2;      // dO half tile (DV / 64 boxes)
+  static constexpr int OBOX = kHalfQ * 128;        // one 64-column box of a half tile
+  static constexpr int SL_Q = 0, SL_O = align1k(QHB), SL_L = SL_O + OHB, SL_D = SL_L + kHalfQ * 4;
+  static constexpr int SLOT = align1k(SL_D + kHalfQ * 4);
   static constexpr int DSB = kKeys * kQT * 2;      // dS^T tile: [2 halves][128 keys][64 queries]
-  // dQ rows staged for the bulk reduce, rows padded by 16 bytes so that the
-  // rows' 16-byte stores of one instruction fall in different banks
-  static constexpr int DQ_ROW = R * 4 + 16;
-  static constexpr int DQB = kQT * DQ_ROW;
+  // dQ tile staged for the TMA reduce-add: softmax warpgroup h stages columns
+  // [h R/2, (h+1) R/2), each warp its 32 rows as one box swizzled over
+  // DQ_SW = 2r bytes (conflict-free row-per-thread stores)
+  static constexpr int DQ_W = R / 2;
+  static constexpr int DQ_SW = DQ_W * 4;
+  static constexpr int DQ_LAYOUT_SHIFT = DQ_SW == 128 ? 0 : (DQ_SW == 64 ? 1 : 2);
+  static constexpr int DQB = kQT * R * 4;
   static constexpr int OFF_K = 0;
   static constexpr int OFF_V = align1k(KB);
-  static constexpr int OFF_ST = OFF_V + VB;
-  static constexpr int OFF_DS = OFF_ST + 2 * STAGE;
-  static constexpr int BASE = OFF_DS + DQB + 256 + 1024;  // without dS tiles; + barriers, alignment slack
-  static constexpr int NDS = BASE + 2 * DSB <= 227 * 1024 ? 2 : 1;  // dS^T tiles in flight
+  static constexpr int OFF_SL = OFF_V + VB;
+  static constexpr int NSLOT = 4;   // half-tile slots (a fifth, where it fits, measured slower)
+  // without the dS tiles: K, V, the ring, the dQ stage, barriers, alignment slack
+  static constexpr int FIXED = OFF_SL + NSLOT * SLOT + DQB + 256 + 1024;
+  static constexpr int NDS = FIXED + 2 * DSB <= 227 * 1024 ? 2 : 1;   // dS^T tiles in flight
+  static constexpr int OFF_DS = OFF_SL + NSLOT * SLOT;
   static constexpr int OFF_DQ = OFF_DS + NDS * DSB;
   static constexpr int OFF_BAR = OFF_DQ + DQB;
   // at least 116 KB so that one CTA (and its 512 TMEM columns) sits on an SM alone
   static constexpr int SMEM = std::max(OFF_BAR + 256 + 1024, 116 * 1024);
   static_assert(OFF_BAR + 256 + 1024 <= 227 * 1024, "shared memory");
   // TMEM columns
-  static constexpr int T_S = 0;          // + 128 h: S^T_h (P^T_h packed in its first 32)
+  static constexpr int T_S = 0;          // + 128 h: S^T_h
   static constexpr int T_DP = 64;        // + 128 h: dP^T_h
   static constexpr int T_DV = 256, T_DK = 256 + DV, T_DQ = 256 + DV + R;
   static_assert(T_DQ + R <= kTmemColsTc, "TMEM columns");
+  static constexpr bool P_OWN = T_DQ + R + 2 * (kHalfQ / 2) <= kTmemColsTc;  // P^T in columns of its own
+  static constexpr int T_P = P_OWN ? T_DQ + R : T_S;   // + (P_OWN ? 32 : 128) h: P^T_h
+  static constexpr int P_STRIDE = P_OWN ? kHalfQ / 2 : 128;
+  // With P^T in its own columns and two dS tiles, the next tile's scores of a
+  // half are issued as soon as the half's softmax warps have read S / dP into
+  // registers, and a tile's dQ product one step later; otherwise the products
+  // follow the softmax of each half.
+  static constexpr bool EARLY = P_OWN && NDS == 2;
   // instruction descriptors
   static constexpr uint32_t ID_S = instr_desc(kKeys, kHalfQ, false);       // S^T, dP^T
   static constexpr uint32_t ID_DV = instr_desc(kKeys, DV, true);           // A = P^T (TMEM), B = dO MN-major
@@ -98,13 +119,16 @@ struct TCfg {
 };
 
 struct TcMaps {
-  CUtensorMap q, k, v, d_out;
+  CUtensorMap q, k, v, d_out, dq;
 };
 
-__device__ __forceinline__ void bulk_reduce_add_f32(float* gdst, const void* ssrc, uint32_t bytes) {
-  asm volatile("cp.reduce.async.bulk.global.shared::cta.bulk_group.add.f32 [%0], [%1], %2;" ::"l"(gdst),
-               "r"(smem_addr(ssrc)), "r"(bytes)
-               : "memory");
+// TMA tensor reduce-add of a shared-memory box into global memory (bulk group).
+__device__ __forceinline__ void tma_reduce_add_3d(const CUtensorMap* map, const void* src, int x, int y, int z) {
+  asm volatile(
+      "cp.reduce.async.bulk.tensor.3d.global.shared::cta.add.tile.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(smem_addr(src)), "r"(x), "r"(y), "r"(z)
+      : "memory");
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read_all() {
@@ -129,17 +153,47 @@ __device__ __forceinline__ void tmem_ld32x2(uint32_t ta, uint32_t tb, uint32_t* 
       : "r"(ta), "r"(tb)
       : "memory");
 }
-// N consecutive 32-bit columns (N = 16, 32 or 64).
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t* v) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : TK_R8(0)
+      : "r"(taddr)
+      : "memory");
+}
+// N consecutive 32-bit columns (N = 8, 16, 32 or 64).
 template <int N>
 __device__ __forceinline__ void tmem_ld_n(uint32_t taddr, uint32_t* v) {
-  if constexpr (N == 16) tmem_ld16(taddr, v);
+  if constexpr (N == 8) tmem_ld8(taddr, v);
+  else if constexpr (N == 16) tmem_ld16(taddr, v);
   else if constexpr (N == 32) tmem_ld32(taddr, v);
   else tmem_ld64(taddr, v);
 }
 
-__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);  // low half = lo
+__device__ __forceinline__ uint32_t pack2(float2 x) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(x.x, x.y);  // low half = x.x
   return *reinterpret_cast<uint32_t*>(&v);
+}
+__device__ __forceinline__ float2 f2(uint32_t a, uint32_t b) {
+  return make_float2(__uint_as_float(a), __uint_as_float(b));
+}
+
+// N TMEM columns (fp32) of this thread's lane, times `mul`, to dst (16-byte aligned).
+template <int N>
+__device__ __forceinline__ void tmem_rows_out(uint32_t taddr, float* dst, float mul, bool store) {
+#pragma unroll
+  for (int c0 = 0; c0 < N; c0 += 32) {
+    constexpr int W = N < 32 ? N : 32;
+    uint32_t v[W];
+    tmem_ld_n<W>(taddr + c0, v);
+    if (store) {
+#pragma unroll
+      for (int c = 0; c < W / 4; ++c)
+        reinterpret_cast<float4*>(dst + c0)[c] =
+            make_float4(__uint_as_float(v[4 * c]) * mul, __uint_as_float(v[4 * c + 1]) * mul,
+                        __uint_as_float(v[4 * c + 2]) * mul, __uint_as_float(v[4 * c + 3]) * mul);
+    }
+  }
 }
 
 template <int R, int DV>
@@ -152,15 +206,17 @@ bwd_tc_kernel(const __grid_constant__ TcMaps maps, const BackwardParams p) {
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
   uint64_t* kv_full = bars + 0;
-  uint64_t* qd_full = bars + 1;      // [2] stage loaded
-  uint64_t* qd_empty = bars + 3;     // [2] stage consumed
-  uint64_t* s_full = bars + 5;       // [2] S^T_h, dP^T_h in TMEM
-  uint64_t* p_ready = bars + 7;      // [2] P^T_h in TMEM, dS^T_h in shared memory
-  uint64_t* ds_free = bars + 9;      // [NDS] dS^T tile read by its last product
-  uint64_t* dq_full = bars + 11;
-  uint64_t* dq_empty = bars + 12;
-  uint64_t* acc_full = bars + 13;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 14);
+  uint64_t* sl_full = bars + 1;      // [NSLOT] half-tile slot loaded
+  uint64_t* sl_empty = bars + 6;     // [NSLOT] half-tile slot consumed
+  uint64_t* s_full = bars + 11;      // [2] S^T_h, dP^T_h in TMEM
+  uint64_t* p_ready = bars + 13;     // [2] P^T_h in TMEM, dS^T_h in shared memory
+  uint64_t* p_free = bars + 15;      // [2] P^T_h read by the dV product (P in its own columns)
+  uint64_t* ds_free = bars + 17;     // [NDS] dS^T tile read by its last product
+  uint64_t* dq_full = bars + 19;
+  uint64_t* dq_empty = bars + 20;
+  uint64_t* acc_full = bars + 21;
+  uint64_t* s_free = bars + 22;      // [2] S^T_h, dP^T_h read into registers (EARLY schedule)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 24);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int S = p.S, G = p.Hq / p.Hkv;
@@ -175,22 +231,29 @@ bwd_tc_kernel(const __grid_constant__ TcMaps maps, const BackwardParams p) {
   const int n_tiles = G * per_head;
   auto tile_head = [&](int t) { return g * G + t / per_head; };
   auto tile_q = [&](int t) { return i0 + t % per_head; };
+  // half tile u = 2 t + h lives in slot u % NSLOT, its (u / NSLOT)-th use of the slot
+  auto slot_of = [](int t, int h) { return (2 * t + h) % C::NSLOT; };
+  auto slot_par = [](int t, int h) { return static_cast<uint32_t>(((2 * t + h) / C::NSLOT) & 1); };
 
   if (tid == 0) {
     mbar_init(kv_full, 1);
+    for (int s = 0; s < C::NSLOT; ++s) {
+      mbar_init(&sl_full[s], 1);
+      mbar_init(&sl_empty[s], 1);
+    }
     for (int s = 0; s < 2; ++s) {
-      mbar_init(&qd_full[s], 1);
-      mbar_init(&qd_empty[s], 1);
       mbar_init(&s_full[s], 1);
       mbar_init(&p_ready[s], 128);
+      mbar_init(&p_free[s], 1);
+      mbar_init(&s_free[s], 128);
     }
     for (int s = 0; s < NDS; ++s) mbar_init(&ds_free[s], 1);
     mbar_init(dq_full, 1);
-    mbar_init(dq_empty, 128);
+    mbar_init(dq_empty, 256);
     mbar_init(acc_full, 1);
     fence_barrier_init();
   }
-  if (warp == 13) {
+  if (warp == 8) {
     tmem_alloc(tmem_slot, kTmemColsTc);
     tmem_relinquish();
   }
@@ -198,7 +261,7 @@ bwd_tc_kernel(const __grid_constant__ TcMaps maps, const BackwardParams p) {
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 12) {
+  if (warp == 9) {
     // ------------------------------------------------------------------ TMA producer
     if (lane == 0) {
       const int kv_plane = b * p.Hkv + g;
@@ -211,220 +274,274 @@ bwd_tc_kernel(const __grid_constant__ TcMaps maps, const BackwardParams p) {
       for (int x = 0; x < DV / 64; ++x)
         tma_load_3d(smem + C::OFF_V + x * kBoxB, &maps.v, 64 * x, j * kKeys, kv_plane, kv_full);
       int issued = 0;
-      for (int t = 0; t < n_tiles; ++t) {
-        const int st = t & 1;
-        if (t >= 2 && !mbar_wait(&qd_empty[st], ((t >> 1) - 1) & 1, p.err)) break;
-        const int bh = b * p.Hq + tile_head(t), i = tile_q(t);
-        unsigned char* sb = smem + C::OFF_ST + st * C::STAGE;
-        mbar_arrive_expect_tx(&qd_full[st], C::QB + C::OB + 2 * kQT * 4);
-        tma_load_3d(sb + C::ST_Q, &maps.q, 0, i * kQT, bh, &qd_full[st]);
+      for (int u = 0; u < 2 * n_tiles; ++u) {
+        const int sl = u % C::NSLOT;
+        if (u >= C::NSLOT && !mbar_wait(&sl_empty[sl], ((u / C::NSLOT) - 1) & 1, p.err)) break;
+        const int t = u >> 1, h = u & 1;
+        const int bh = b * p.Hq + tile_head(t), row = tile_q(t) * kQT + h * kHalfQ;
+        unsigned char* sb = smem + C::OFF_SL + sl * C::SLOT;
+        mbar_arrive_expect_tx(&sl_full[sl], C::QHB + C::OHB + 2 * kHalfQ * 4);
+        tma_load_3d(sb + C::SL_Q, &maps.q, 0, row, bh, &sl_full[sl]);
         for (int x = 0; x < DV / 64; ++x)
-          tma_load_3d(sb + C::ST_O + x * kBoxB, &maps.d_out, 64 * x, i * kQT, bh, &qd_full[st]);
-        const size_t srow = static_cast<size_t>(bh) * p.S_pad + static_cast<size_t>(i) * kQT;
-        bulk_g2s(sb + C::ST_LSE, p.lse2 + srow, kQT * 4, &qd_full[st]);
-        bulk_g2s(sb + C::ST_D, p.dsum + srow, kQT * 4, &qd_full[st]);
-        issued = t + 1;
+          tma_load_3d(sb + C::SL_O + x * C::OBOX, &maps.d_out, 64 * x, row, bh, &sl_full[sl]);
+        const size_t srow = static_cast<size_t>(bh) * p.S_pad + row;
+        bulk_g2s(sb + C::SL_L, p.nl2 + srow, kHalfQ * 4, &sl_full[sl]);
+        bulk_g2s(sb + C::SL_D, p.nd + srow, kHalfQ * 4, &sl_full[sl]);
+        issued = u + 1;
       }
       // no copy may still be landing in shared memory when the CTA exits
       // (normally all were consumed; after a timed-out wait, bounded waits)
       mbar_wait(kv_full, 0, p.err);
-      for (int t = std::max(0, issued - 2); t < issued; ++t) mbar_wait(&qd_full[t & 1], (t >> 1) & 1, p.err);
+      for (int u = std::max(0, issued - C::NSLOT); u < issued; ++u)
+        mbar_wait(&sl_full[u % C::NSLOT], (u / C::NSLOT) & 1, p.err);
     }
-  } else if (warp == 13) {
+  } else if (warp == 8) {
     // ------------------------------------------------------------------ MMA issuer
     const uint32_t s_base = smem_addr(smem);
     // one descriptor serves a tile read K-major and MN-major: SBO is the stride of
     // 8-row groups either way, LBO the stride of MN atoms (unused when N fits one)
-    const Desc dK_d = make_desc(s_base + C::OFF_K, 16, 8 * C::QK_SW, C::QK_LAYOUT);     // K
-    const Desc dV_a = make_desc(s_base + C::OFF_V, 16, 1024, 2u);                       // V, K-major
-    const Desc dQ_b = make_desc(s_base + C::OFF_ST + C::ST_Q, 16, 8 * C::QK_SW, C::QK_LAYOUT);     // Q
-    const Desc dO_bk = make_desc(s_base + C::OFF_ST + C::ST_O, 16, 1024, 2u);           // dO, K-major
-    const Desc dO_bm = make_desc(s_base + C::OFF_ST + C::ST_O, kBoxB, 1024, 2u);        // dO, MN-major
-    const Desc dS_ak = make_desc(s_base + C::OFF_DS, 16, 1024, 2u);                     // dS^T, K-major
-    const Desc dS_am = make_desc(s_base + C::OFF_DS, C::DSB / 2, 1024, 2u);             // dS, MN-major
+    const Desc dK_d = make_desc(s_base + C::OFF_K, 16, 8 * C::QK_SW, C::QK_LAYOUT);       // K
+    const Desc dV_a = make_desc(s_base + C::OFF_V, 16, 1024, 2u);                         // V, K-major
+    const Desc dQ_b = make_desc(s_base + C::OFF_SL + C::SL_Q, 16, 8 * C::QK_SW, C::QK_LAYOUT);  // Q_h
+    const Desc dO_bk = make_desc(s_base + C::OFF_SL + C::SL_O, 16, 1024, 2u);             // dO_h, K-major
+    const Desc dO_bm = make_desc(s_base + C::OFF_SL + C::SL_O, C::OBOX, 1024, 2u);        // dO_h, MN-major
+    const Desc dS_ak = make_desc(s_base + C::OFF_DS, 16, 1024, 2u);                       // dS^T, K-major
+    const Desc dS_am = make_desc(s_base + C::OFF_DS, C::DSB / 2, 1024, 2u);               // dS, MN-major
     auto issue_sdp = [&](int t, int h) {   // S^T_h, dP^T_h of tile t
-      const uint32_t so = (t & 1) * C::STAGE;
+      const uint32_t so = slot_of(t, h) * C::SLOT;
 #pragma unroll
       for (int k = 0; k < R / 16; ++k)
-        mma_ss_e(tmem + C::T_S + 128 * h, dK_d.at(k * 32), dQ_b.at(so + h * kHalfQ * C::QK_SW + k * 32),
-                 C::ID_S, k > 0);
+        mma_ss_e(tmem + C::T_S + 128 * h, dK_d.at(k * 32), dQ_b.at(so + k * 32), C::ID_S, k > 0);
 #pragma unroll
-      for (int k = 0; k < DV / 16; ++k) {
-        const uint32_t ko = (k / 4) * kBoxB + (k % 4) * 32;
-        mma_ss_e(tmem + C::T_DP + 128 * h, dV_a.at(ko), dO_bk.at(so + ko + h * kHalfQ * 128), C::ID_S, k > 0);
-      }
+      for (int k = 0; k < DV / 16; ++k)
+        mma_ss_e(tmem + C::T_DP + 128 * h, dV_a.at((k / 4) * kBoxB + (k % 4) * 32),
+                 dO_bk.at(so + (k / 4) * C::OBOX + (k % 4) * 32), C::ID_S, k > 0);
       tc_commit_e(&s_full[h]);
     };
-    auto issue_dvdk = [&](int t, int h) {  // dV += P^T_h dO_h, dK += dS^T_h Q_h
-      const uint32_t so = (t & 1) * C::STAGE;
+    auto issue_dvdk = [&](int t, int h) {  // dV += P^T_h dO_h, dK += dS^T_h Q_h; the slot is then free
+      const uint32_t so = slot_of(t, h) * C::SLOT;
       const uint32_t dso = (t % NDS) * C::DSB + h * (C::DSB / 2);
 #pragma unroll
       for (int kk = 0; kk < kHalfQ / 16; ++kk)
-        mma_ts_e(tmem + C::T_DV, tmem + C::T_S + 128 * h + 8 * kk,
-                 dO_bm.at(so + (h * kHalfQ + 16 * kk) * 128), C::ID_DV, (t > 0 || h > 0 || kk > 0) ? 1u : 0u);
+        mma_ts_e(tmem + C::T_DV, tmem + C::T_P + C::P_STRIDE * h + 8 * kk, dO_bm.at(so + 16 * kk * 128),
+                 C::ID_DV, (t > 0 || h > 0 || kk > 0) ? 1u : 0u);
+      if (C::P_OWN) tc_commit_e(&p_free[h]);
 #pragma unroll
       for (int kk = 0; kk < kHalfQ / 16; ++kk)
-        mma_ss_e(tmem + C::T_DK, dS_ak.at(dso + kk * 32),
-                 dQ_b.at(so + (h * kHalfQ + 16 * kk) * C::QK_SW), C::ID_DK, (t > 0 || h > 0 || kk > 0) ? 1u : 0u);
+        mma_ss_e(tmem + C::T_DK, dS_ak.at(dso + kk * 32), dQ_b.at(so + 16 * kk * C::QK_SW), C::ID_DK,
+                 (t > 0 || h > 0 || kk > 0) ? 1u : 0u);
+      tc_commit_e(&sl_empty[slot_of(t, h)]);
     };
-    bool ok = __all_sync(0xffffffffu, mbar_wait(kv_full, 0, p.err) && mbar_wait(&qd_full[0], 0, p.err));
+    auto issue_dq = [&](int t) {           // dQ_t = dS K over the 128 keys
+      const uint32_t dso = (t % NDS) * C::DSB;
+#pragma unroll
+      for (int k = 0; k < kKeys / 16; ++k)
+        mma_ss_e(tmem + C::T_DQ, dS_am.at(dso + k * 16 * 128), dK_d.at(k * 16 * C::QK_SW), C::ID_DQ, k > 0);
+      tc_commit_e(dq_full);
+      tc_commit_e(&ds_free[t % NDS]);
+    };
+    auto wait_all = [&](uint64_t* bar, uint32_t parity) {
+      return __all_sync(0xffffffffu, mbar_wait(bar, parity, p.err));
+    };
+    bool ok = wait_all(kv_full, 0) && wait_all(&sl_full[0], 0);
     if (ok) {
       tc_fence_after();
       issue_sdp(0, 0);
-      issue_sdp(0, 1);
+      ok = wait_all(&sl_full[1], 0);
+      tc_fence_after();
+      if (ok) issue_sdp(0, 1);
     }
-    for (int t = 0; ok && t < n_tiles; ++t) {
-      const bool next = t + 1 < n_tiles;
-      if (!(ok = __all_sync(0xffffffffu, mbar_wait(&p_ready[0], t & 1, p.err)))) break;
-      tc_fence_after();
-      issue_dvdk(t, 0);
-      if (next) {
-        if (!(ok = __all_sync(0xffffffffu, mbar_wait(&qd_full[(t + 1) & 1], ((t + 1) >> 1) & 1, p.err)))) break;
+    if constexpr (C::EARLY) {
+      // per tile and half: the next tile's scores as soon as the half's softmax
+      // warps release S / dP, then (half 0) the previous tile's dQ product, then
+      // this tile's dV / dK products when P / dS arrive
+      for (int t = 0; ok && t < n_tiles; ++t) {
+        for (int h = 0; ok && h < 2; ++h) {
+          if (t + 1 < n_tiles) {
+            if (!(ok = wait_all(&s_free[h], t & 1) && wait_all(&sl_full[slot_of(t + 1, h)], slot_par(t + 1, h))))
+              break;
+            tc_fence_after();
+            issue_sdp(t + 1, h);
+          }
+          if (h == 0 && t > 0) {
+            if (t > 1 && !(ok = wait_all(dq_empty, (t - 2) & 1))) break;
+            tc_fence_after();
+            issue_dq(t - 1);
+          }
+          if (!(ok = wait_all(&p_ready[h], t & 1))) break;
+          tc_fence_after();
+          issue_dvdk(t, h);
+        }
+      }
+      if (ok && n_tiles > 1) ok = wait_all(dq_empty, (n_tiles - 2) & 1);
+      if (ok) {
         tc_fence_after();
-        issue_sdp(t + 1, 0);
+        issue_dq(n_tiles - 1);
       }
-      if (!(ok = __all_sync(0xffffffffu, mbar_wait(&p_ready[1], t & 1, p.err)))) break;
-      tc_fence_after();
-      issue_dvdk(t, 1);
-      if (t > 0 && !(ok = __all_sync(0xffffffffu, mbar_wait(dq_empty, (t - 1) & 1, p.err)))) break;
-      tc_fence_after();
-      {  // dQ_t = dS K over the 128 keys
-        const uint32_t dso = (t % NDS) * C::DSB;
-#pragma unroll
-        for (int k = 0; k < kKeys / 16; ++k)
-          mma_ss_e(tmem + C::T_DQ, dS_am.at(dso + k * 16 * 128), dK_d.at(k * 16 * C::QK_SW), C::ID_DQ, k > 0);
+    } else {
+      for (int t = 0; ok && t < n_tiles; ++t) {
+        const bool next = t + 1 < n_tiles;
+        for (int h = 0; ok && h < 2; ++h) {
+          if (!(ok = wait_all(&p_ready[h], t & 1))) break;
+          if (next && !(ok = wait_all(&sl_full[slot_of(t + 1, h)], slot_par(t + 1, h)))) break;
+          tc_fence_after();
+          // P^T_h in columns of its own: the next tile's scores of this half go
+          // first; otherwise P^T_h overlays S^T_h and its dV product goes first
+          if (C::P_OWN && next) issue_sdp(t + 1, h);
+          issue_dvdk(t, h);
+          if (h == 1) {
+            // dQ before the next tile's half-1 scores: with one dS tile the next
+            // tile's half-0 dS waits for it
+            if (t > 0 && !(ok = wait_all(dq_empty, (t - 1) & 1))) break;
+            tc_fence_after();
+            issue_dq(t);
+          }
+          if (!C::P_OWN && next) issue_sdp(t + 1, h);
+        }
       }
-      tc_commit_e(dq_full);
-      tc_commit_e(&ds_free[t % NDS]);
-      tc_commit_e(&qd_empty[t & 1]);
-      if (next) issue_sdp(t + 1, 1);
     }
     if (ok) tc_commit_e(acc_full);
-  } else if (warp < 8) {
+  } else {
     // ------------------------------------------------------------------ softmax gradient warps
     const int h = warp >> 2;                      // query half
     const int kt = (warp & 3) * 32 + lane;        // key of this thread within the tile (TMEM lane)
     const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
     const uint32_t tS = tmem + C::T_S + 128 * h + lane_off, tD = tmem + C::T_DP + 128 * h + lane_off;
+    const uint32_t tP = tmem + C::T_P + C::P_STRIDE * h + lane_off;
     const bool kvalid = j * kKeys + kt < S;
     const float sl2 = p.scale * 1.4426950408889634f;
-    for (int t = 0; t < n_tiles; ++t) {
-      const int st = t & 1, buf = t % NDS;
-      bool ok = mbar_wait(&s_full[h], t & 1, p.err) && mbar_wait(&qd_full[st], (t >> 1) & 1, p.err);
-      if (ok && t >= NDS) ok = mbar_wait(&ds_free[buf], ((t / NDS) - 1) & 1, p.err);
-      if (!__all_sync(0xffffffffu, ok)) break;
-      tc_fence_after();
-      const unsigned char* sb = smem + C::OFF_ST + st * C::STAGE;
-      const float* lse2 = reinterpret_cast<const float*>(sb + C::ST_LSE) + h * kHalfQ;
-      const float* dsum = reinterpret_cast<const float*>(sb + C::ST_D) + h * kHalfQ;
-      unsigned char* ds_row = smem + C::OFF_DS + buf * C::DSB + h * (C::DSB / 2) + kt * 128;
-      // keys past S, and keys after the query on the diagonal tile, get weight 0
-      const int qlim = (p.causal && tile_q(t) == j) ? kt - h * kHalfQ : 0;  // visible iff column >= qlim
-      // warp-uniform choice: both paths issue warp-collective TMEM loads and stores
-      const bool masked = __any_sync(0xffffffffu, !kvalid || qlim > 0);
-      auto chunk = [&](auto mask_tag, int c) {
-        constexpr bool kMask = decltype(mask_tag)::value;
-        uint32_t v[64];   // [0, 32): S^T, [32, 64): dP^T
-        tmem_ld32x2(tS + 32 * c, tD + 32 * c, v);
-        uint32_t pk[16], dk[16];
-#pragma unroll
-        for (int e2 = 0; e2 < 16; ++e2) {
-          float pr[2], dsv[2];
-#pragma unroll
-          for (int u = 0; u < 2; ++u) {
-            const int e = 2 * e2 + u, col = 32 * c + e;
-            float x = __uint_as_float(v[e]) * sl2 - lse2[col];
-            if (kMask && (!kvalid || col < qlim)) x = -INFINITY;
-            pr[u] = fast_exp2(x);
-            dsv[u] = pr[u] * (__uint_as_float(v[32 + e]) - dsum[col]);
-          }
-          pk[e2] = pack2(pr[0], pr[1]);
-          dk[e2] = pack2(dsv[0], dsv[1]);
-        }
-        tmem_st16(tS + 16 * c, pk);
-        // dS^T row kt, queries 32c .. 32c+31 of the half: four 16-byte chunks, SW128 swizzle
-#pragma unroll
-        for (int m = 0; m < 4; ++m) {
-          const int chunk_i = (4 * c + m) ^ (kt & 7);
-          *reinterpret_cast<uint4*>(ds_row + chunk_i * 16) =
-              make_uint4(dk[4 * m], dk[4 * m + 1], dk[4 * m + 2], dk[4 * m + 3]);
-        }
-      };
-#pragma unroll
-      for (int c = 0; c < kHalfQ / 32; ++c) {
-        if (masked) chunk(std::true_type{}, c);
-        else chunk(std::false_type{}, c);
+    const float2 sl2x2 = make_float2(sl2, sl2);
+    bool ok = true, pending = false;
+    // dQ of tile t (thread kt: query kt of the tile), columns [h R/2, (h+1) R/2):
+    // read from TMEM after the next tile's softmax (dq_fetch), then staged in
+    // shared memory and added into global dq by a TMA reduce per warp (its 32
+    // rows), so that no warp waits for another (dq_store).
+    unsigned char* dq_box = smem + C::OFF_DQ + h * (kQT * C::DQ_SW) + (warp & 3) * (32 * C::DQ_SW);
+    uint32_t wq[C::DQ_W];
+    bool dq_ok = false;
+    auto dq_fetch = [&](int t) {
+      dq_ok = __all_sync(0xffffffffu, ok && mbar_wait(dq_full, t & 1, p.err));
+      if (dq_ok) {
+        tc_fence_after();
+        tmem_ld_n<C::DQ_W>(tmem + C::T_DQ + h * C::DQ_W + lane_off, wq);
+        tc_fence_before();
+        mbar_arrive(dq_empty);
       }
-      tmem_wait_st();
-      fence_proxy_async_smem();
-      tc_fence_before();
-      mbar_arrive(&p_ready[h]);
-    }
-  } else {
-    // ------------------------------------------------------------------ dQ / dK / dV epilogue
-    const int row = (warp & 3) * 32 + lane;       // TMEM lane: a query (dQ) or a key (dK, dV)
-    const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
-    float* stage = reinterpret_cast<float*>(smem + C::OFF_DQ + row * C::DQ_ROW);
-    bool ok = true;
-    bool pending = false;
-    for (int t = 0; t < n_tiles; ++t) {
-      ok = mbar_wait(dq_full, t & 1, p.err);
-      if (!__all_sync(0xffffffffu, ok)) { ok = false; break; }
-      tc_fence_after();
-      uint32_t v[R];
-      tmem_ld_n<R>(tmem + C::T_DQ + lane_off, v);
-      tc_fence_before();
-      mbar_arrive(dq_empty);
-      const int i = tile_q(t);
-      const int q = i * kQT + row;
-      if (q < S) {
-        if (pending) bulk_wait_read_all();   // the previous row's reduce has read the stage
+    };
+    auto dq_store = [&](int t) {
+      const int row0 = tile_q(t) * kQT + (warp & 3) * 32;   // first query of this warp's rows
+      if (dq_ok && row0 < S) {
+        if (lane == 0 && pending) bulk_wait_read_all();   // the previous reduce has read the box
+        __syncwarp();
 #pragma unroll
-        for (int c = 0; c < R / 4; ++c)
-          reinterpret_cast<float4*>(stage)[c] =
-              make_float4(__uint_as_float(v[4 * c]) * p.scale, __uint_as_float(v[4 * c + 1]) * p.scale,
-                          __uint_as_float(v[4 * c + 2]) * p.scale, __uint_as_float(v[4 * c + 3]) * p.scale);
+        for (int c = 0; c < C::DQ_SW / 16; ++c) {
+          const int pc = c ^ ((lane >> C::DQ_LAYOUT_SHIFT) & (C::DQ_SW / 16 - 1));
+          *reinterpret_cast<float4*>(dq_box + lane * C::DQ_SW + pc * 16) =
+              make_float4(__uint_as_float(wq[4 * c]) * p.scale, __uint_as_float(wq[4 * c + 1]) * p.scale,
+                          __uint_as_float(wq[4 * c + 2]) * p.scale, __uint_as_float(wq[4 * c + 3]) * p.scale);
+        }
         fence_proxy_async_smem();
-        const size_t x = (static_cast<size_t>(b) * p.Hq + tile_head(t)) * S + q;
-        bulk_reduce_add_f32(p.dq + x * R, stage, R * 4);
-        bulk_commit();
-        pending = true;
+        __syncwarp();
+        if (lane == 0) {
+          tma_reduce_add_3d(&maps.dq, dq_box, h * C::DQ_W, row0, b * p.Hq + tile_head(t));
+          bulk_commit();
+          pending = true;
+        }
       }
+      if (!dq_ok) ok = false;
+      dq_ok = false;
+    };
+    for (int t = 0; t < n_tiles; ++t) {
+      const int sl = slot_of(t, h), buf = t % NDS;
+      if (ok) {
+        ok = mbar_wait(&s_full[h], t & 1, p.err) && mbar_wait(&sl_full[sl], slot_par(t, h), p.err);
+        if (ok && t >= NDS) ok = mbar_wait(&ds_free[buf], ((t / NDS) - 1) & 1, p.err);
+        ok = __all_sync(0xffffffffu, ok);
+      }
+      if (ok) {
+        tc_fence_after();
+        const unsigned char* sb = smem + C::OFF_SL + sl * C::SLOT;
+        const float* nl2 = reinterpret_cast<const float*>(sb + C::SL_L);
+        const float* nd = reinterpret_cast<const float*>(sb + C::SL_D);
+        unsigned char* ds_row = smem + C::OFF_DS + buf * C::DSB + h * (C::DSB / 2) + kt * 128;
+        // keys past S, and keys after the query on the diagonal tile, get weight 0
+        const int qlim = (p.causal && tile_q(t) == j) ? kt - h * kHalfQ : 0;  // visible iff column >= qlim
+        // warp-uniform choice: both paths issue warp-collective TMEM loads and stores
+        const bool masked = __any_sync(0xffffffffu, !kvalid || qlim > 0);
+        auto chunk = [&](auto mask_tag, int c) {
+          constexpr bool kMask = decltype(mask_tag)::value;
+          uint32_t v[64];   // [0, 32): S^T, [32, 64): dP^T
+          tmem_ld32x2(tS + 32 * c, tD + 32 * c, v);
+          if (C::EARLY && c == kHalfQ / 32 - 1) {   // S^T_h, dP^T_h may be overwritten
+            tc_fence_before();
+            mbar_arrive(&s_free[h]);
+          }
+          uint32_t pk[16], dk[16];
+#pragma unroll
+          for (int e2 = 0; e2 < 16; ++e2) {
+            const int col = 32 * c + 2 * e2;
+            float2 x = ffma2(f2(v[2 * e2], v[2 * e2 + 1]), sl2x2, *reinterpret_cast<const float2*>(nl2 + col));
+            if (kMask) {
+              if (!kvalid || col < qlim) x.x = -INFINITY;
+              if (!kvalid || col + 1 < qlim) x.y = -INFINITY;
+            }
+            const float2 pr = make_float2(fast_exp2(x.x), fast_exp2(x.y));
+            const float2 dsv = fmul2(pr, fadd2(f2(v[32 + 2 * e2], v[33 + 2 * e2]),
+                                               *reinterpret_cast<const float2*>(nd + col)));
+            pk[e2] = pack2(pr);
+            dk[e2] = pack2(dsv);
+          }
+          // P^T_h may overwrite the previous tile's only once its dV product has read it
+          if (C::P_OWN && c == 0 && t > 0) {
+            const bool okp = mbar_wait(&p_free[h], (t - 1) & 1, p.err);
+            if (!__all_sync(0xffffffffu, okp)) ok = false;
+          }
+          tmem_st16(tP + 16 * c, pk);
+          // dS^T row kt, queries 32c .. 32c+31 of the half: four 16-byte chunks, SW128 swizzle
+#pragma unroll
+          for (int m = 0; m < 4; ++m) {
+            const int chunk_i = (4 * c + m) ^ (kt & 7);
+            *reinterpret_cast<uint4*>(ds_row + chunk_i * 16) =
+                make_uint4(dk[4 * m], dk[4 * m + 1], dk[4 * m + 2], dk[4 * m + 3]);
+          }
+        };
+#pragma unroll
+        for (int c = 0; c < kHalfQ / 32; ++c) {
+          if (masked) chunk(std::true_type{}, c);
+          else chunk(std::false_type{}, c);
+        }
+        tmem_wait_st();
+        fence_proxy_async_smem();
+        tc_fence_before();
+        mbar_arrive(&p_ready[h]);
+      }
+      if (t > 0) {
+        dq_fetch(t - 1);
+        dq_store(t - 1);
+      }
+    }
+    if (n_tiles > 0) {
+      dq_fetch(n_tiles - 1);
+      dq_store(n_tiles - 1);
     }
     if (pending) bulk_wait_all();
     if (ok) ok = mbar_wait(acc_full, 0, p.err);
     if (__all_sync(0xffffffffu, ok)) {
       tc_fence_after();
-      const int key = j * kKeys + row;
+      const int key = j * kKeys + kt;
       const size_t kx = (static_cast<size_t>(b) * p.Hkv + g) * S + key;
-      {
-        uint32_t v[R];
-        tmem_ld_n<R>(tmem + C::T_DK + lane_off, v);
-        if (key < S) {
-          float4* dst = reinterpret_cast<float4*>(p.dk + kx * R);
-#pragma unroll
-          for (int c = 0; c < R / 4; ++c)
-            dst[c] = make_float4(__uint_as_float(v[4 * c]) * p.scale, __uint_as_float(v[4 * c + 1]) * p.scale,
-                                 __uint_as_float(v[4 * c + 2]) * p.scale, __uint_as_float(v[4 * c + 3]) * p.scale);
-        }
-      }
-#pragma unroll
-      for (int c0 = 0; c0 < DV / 32; ++c0) {
-        uint32_t v[32];
-        tmem_ld32(tmem + C::T_DV + lane_off + 32 * c0, v);
-        if (key < S) {
-          float4* dst = reinterpret_cast<float4*>(p.dv + kx * DV + 32 * c0);
-#pragma unroll
-          for (int c = 0; c < 8; ++c)
-            dst[c] = make_float4(__uint_as_float(v[4 * c]), __uint_as_float(v[4 * c + 1]),
-                                 __uint_as_float(v[4 * c + 2]), __uint_as_float(v[4 * c + 3]));
-        }
+      const bool store = key < S;
+      if (h == 0) {
+        tmem_rows_out<R>(tmem + C::T_DK + lane_off, p.dk + kx * R, p.scale, store);
+        tmem_rows_out<DV / 2>(tmem + C::T_DV + lane_off, p.dv + kx * DV, 1.f, store);
+      } else {
+        tmem_rows_out<DV / 2>(tmem + C::T_DV + DV / 2 + lane_off, p.dv + kx * DV + DV / 2, 1.f, store);
       }
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 13) {
+  if (warp == 8) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemColsTc);
   }
@@ -434,10 +551,11 @@ template <int R, int DV>
 cudaError_t launch_tc(const BackwardParams& p, cudaStream_t stream) {
   using C = TCfg<R, DV>;
   TcMaps maps;
-  if (!make_map(&maps.q, p.q, R, p.S, p.B * p.Hq, R, kQT, C::QK_SW) ||
+  if (!make_map(&maps.q, p.q, R, p.S, p.B * p.Hq, R, kHalfQ, C::QK_SW) ||
       !make_map(&maps.k, p.k, R, p.S, p.B * p.Hkv, R, kKeys, C::QK_SW) ||
       !make_map(&maps.v, p.v, DV, p.S, p.B * p.Hkv, 64, kKeys, 128) ||
-      !make_map(&maps.d_out, p.d_out, DV, p.S, p.B * p.Hq, 64, kQT, 128))
+      !make_map(&maps.d_out, p.d_out, DV, p.S, p.B * p.Hq, 64, kHalfQ, 128) ||
+      !make_map(&maps.dq, p.dq, R, p.S, p.B * p.Hq, C::DQ_W, 32, C::DQ_SW, true))
     return cudaErrorInvalidValue;
   auto kern = bwd_tc_kernel<R, DV>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);

@@ -113,9 +113,10 @@ struct BackwardParams {
   float* dq;          // fp32 [B][Hq][S][R]  (accumulated: zeroed by the preprocessing kernel)
   float* dk;          // fp32 [B][Hkv][S][R]
   float* dv;          // fp32 [B][Hkv][S][DV]
-  // workspace, rows padded to S_pad (a multiple of 128) per (b, query head):
-  float* lse2;        // [B*Hq][S_pad] lse * log2(e); +inf on rows >= S (weight 0)
-  float* dsum;        // [B*Hq][S_pad] rowsum(d_out * out); 0 on rows >= S
+  // workspace, rows padded to S_pad (a multiple of 128) per (b, query head),
+  // both negated so that the kernels add them:
+  float* nl2;         // [B*Hq][S_pad] -lse * log2(e); -inf on rows >= S (weight 0)
+  float* nd;          // [B*Hq][S_pad] -rowsum(d_out * out); 0 on rows >= S
   int* err;
   int B, Hq, Hkv, S, S_pad, R, DV;
   int causal;

@@ -54,14 +54,6 @@ __device__ __forceinline__ float max3f(float a, float b, float c) {
   return r;
 }
 
-__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
-  uint64_t d;
-  asm("add.rn.f32x2 %0, %1, %2;"
-      : "=l"(d)
-      : "l"(*reinterpret_cast<uint64_t*>(&a)), "l"(*reinterpret_cast<uint64_t*>(&b)));
-  return *reinterpret_cast<float2*>(&d);
-}
-
 // Maximum of 128 floats held in registers (three-input max tree, few temporaries).
 __device__ __forceinline__ float max128(const uint32_t* v) {
 #define TK_F(i) __uint_as_float(v[i])

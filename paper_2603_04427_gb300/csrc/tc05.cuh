@@ -218,23 +218,25 @@ inline PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// 3-D bf16 map over [planes][rows][inner] with a (box_inner x box_rows x 1) box.
+// 3-D map over [planes][rows][inner] (bf16, or fp32 when f32) with a
+// (box_inner x box_rows x 1) box.
 inline bool make_map(CUtensorMap* m, const void* base, int inner, int rows, int planes, int box_inner,
-              int box_rows, int swizzle_bytes) {
+                     int box_rows, int swizzle_bytes, bool f32 = false) {
   auto enc = encode_fn();
   if (!enc) return false;
+  const cuuint64_t es = f32 ? 4 : 2;
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows),
                         static_cast<cuuint64_t>(planes)};
-  cuuint64_t strides[2] = {static_cast<cuuint64_t>(inner) * 2,
-                           static_cast<cuuint64_t>(inner) * rows * 2};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(inner) * es,
+                           static_cast<cuuint64_t>(inner) * rows * es};
   cuuint32_t box[3] = {static_cast<cuuint32_t>(box_inner), static_cast<cuuint32_t>(box_rows), 1};
   cuuint32_t estr[3] = {1, 1, 1};
   CUtensorMapSwizzle sw = swizzle_bytes == 32   ? CU_TENSOR_MAP_SWIZZLE_32B
                           : swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
                                                 : CU_TENSOR_MAP_SWIZZLE_128B;
-  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
-             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
-             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  return enc(m, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+             const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace tk

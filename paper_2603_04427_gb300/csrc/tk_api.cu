@@ -177,7 +177,7 @@ tk_status tk_attn_forward(const void* q, const void* k, const void* v, void* out
 
 size_t tk_backward_workspace_size(int32_t batch, int32_t h_q, int32_t seq) {
   if (batch < 0 || h_q <= 0 || seq < 0) return 0;
-  // two float arrays (lse * log2 e and rowsum(d_out * out)) of backward_rows(seq) per (b, h)
+  // two float arrays (-lse log2 e and -rowsum(d_out * out)) of backward_rows(seq) per (b, h)
   return 2 * ((static_cast<size_t>(batch) * h_q * tk::backward_rows(seq) * 4 + 255) / 256 * 256);
 }
 
@@ -210,8 +210,8 @@ tk_status tk_attn_backward(const void* q, const void* k, const void* v, const vo
   p.dq = dq; p.dk = dk; p.dv = dv; p.err = dev->err;
   p.S_pad = tk::backward_rows(seq);
   const size_t half = need / 2;   // each array 256-byte aligned
-  p.lse2 = static_cast<float*>(workspace);
-  p.dsum = reinterpret_cast<float*>(static_cast<unsigned char*>(workspace) + half);
+  p.nl2 = static_cast<float*>(workspace);
+  p.nd = reinterpret_cast<float*>(static_cast<unsigned char*>(workspace) + half);
   p.B = batch; p.Hq = h_q; p.Hkv = h_kv; p.S = seq; p.R = r; p.DV = d_v;
   p.causal = causal != 0;
   p.scale = scale;
