@@ -156,8 +156,9 @@ tk_status tk_attn_forward(const void* q, const void* k, const void* v, void* out
                           int32_t seq, int32_t r, int32_t d_v, float scale, int32_t causal,
                           void* stream);
 
-/* Bytes of workspace tk_attn_backward needs (one float per query row, rounded
- * up); 0 for invalid arguments.                                             */
+/* Bytes of workspace tk_attn_backward needs: two floats per query row (each
+ * row's -lse log2 e and -rowsum(d_out * out)), rows padded to a multiple of
+ * 128 per (sequence, query head); 0 for invalid arguments.                  */
 size_t tk_backward_workspace_size(int32_t batch, int32_t h_q, int32_t seq);
 
 /* Gradients of prefill attention (the training path of thin-key attention;
@@ -175,8 +176,9 @@ size_t tk_backward_workspace_size(int32_t batch, int32_t h_q, int32_t seq);
  *   workspace: tk_backward_workspace_size bytes, 256-byte aligned (scratch)
  *   scale, causal: as in the forward.
  * The products run on the tensor cores with bf16 operands (P and dS rounded
- * to bf16) and fp32 accumulation; dq is accumulated across key tiles with
- * fp32 atomic adds, so its low bits may vary run to run.                    */
+ * to bf16) and fp32 accumulation (tcgen05 for r <= 64, mma.sync for
+ * r = 128); dq is accumulated across key tiles with fp32 reduce-adds, so its
+ * low bits may vary run to run.  Two launches (preprocessing, gradients).    */
 tk_status tk_attn_backward(const void* q, const void* k, const void* v, const void* out,
                            const void* d_out, const float* lse, float* dq, float* dk, float* dv,
                            void* workspace, size_t workspace_bytes, int32_t batch, int32_t h_q,
