@@ -633,11 +633,11 @@ def main():
             pf.update(frac=pf["tflops"] / peaks["bf16_tflops"], peak=peaks["bf16_tflops"],
                       peak_source=peak_src, bound="tensor",
                       traffic=recorded_traffic("prefill", pw.name,
-                                               source_hash("prefill.cu", "common.cuh")))
+                                               source_hash("prefill.cu", "common.cuh", "tc05.cuh")))
         extra[pw.name] = dict(pw.as_config(), **pf)
         bw = measure_backward(pw, 10, device, torch)
         bw.update(frac=bw["tflops"] / peaks["bf16_tflops"], peak=peaks["bf16_tflops"],
-                  peak_source=peak_src, bound="tensor", kernel="mma.sync m16n8k16")
+                  peak_source=peak_src, bound="tensor", kernel="bwd_tc_kernel<32,128> (tcgen05)")
         extra[pw.name.replace("prefill", "backward")] = dict(pw.as_config(), **bw)
         cw = wl.CHUNKED_PREFILL
         cp = measure_chunked_prefill(cw, 20, device, torch)

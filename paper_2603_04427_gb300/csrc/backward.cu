@@ -110,38 +110,44 @@ __device__ __forceinline__ void load_tile(uint32_t dst, const unsigned char* src
 }
 
 // ---------------------------------------------------------------- preprocessing
-// One warp per padded statistics row (b, h, i < S_pad): for i < S,
-// nd = -sum_c dO * out (fp32), nl2 = -lse * log2(e) and the row of dQ zeroed;
-// for S <= i < S_pad, nd = 0 and nl2 = -inf (such rows get softmax weight 0).
+// DV / 8 threads per padded statistics row (b, h, i < S_pad), 16 bytes of out
+// and of d_out each: for i < S, nd = -sum_c dO * out (fp32), nl2 = -lse *
+// log2(e) and the row of dQ zeroed; for S <= i < S_pad, nd = 0 and nl2 = -inf
+// (such rows get softmax weight 0).
+constexpr int kPrepThreads = 256;
 template <int R, int DV>
-__global__ void __launch_bounds__(256) bwd_prep(const BackwardParams p) {
-  const long long row = static_cast<long long>(blockIdx.x) * 8 + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
+__global__ void __launch_bounds__(kPrepThreads) bwd_prep(const BackwardParams p) {
+  constexpr int TPR = DV / 8;                       // threads per row
+  constexpr int RPB = kPrepThreads / TPR;           // rows per block
+  static_assert(32 % TPR == 0, "a row's threads sit in one warp");
+  const int sub = threadIdx.x % TPR;
+  const long long row = static_cast<long long>(blockIdx.x) * RPB + threadIdx.x / TPR;
   const long long rows = static_cast<long long>(p.B) * p.Hq * p.S_pad;
-  if (row >= rows) return;
-  const long long bh = row / p.S_pad;
-  const int i = static_cast<int>(row - bh * p.S_pad);
-  if (i >= p.S) {
-    if (lane == 0) {
-      p.nd[row] = 0.f;
-      p.nl2[row] = -INFINITY;
-    }
-    return;
-  }
+  // no lane leaves before the shuffle below: a warp holds several rows
+  const bool in_grid = row < rows;
+  const long long bh = in_grid ? row / p.S_pad : 0;
+  const int i = in_grid ? static_cast<int>(row - bh * p.S_pad) : 0;
+  const bool real = in_grid && i < p.S;
   const long long x = bh * p.S + i;   // row of the [B][Hq][S] tensors
-  const __nv_bfloat16* o = static_cast<const __nv_bfloat16*>(p.out) + x * DV;
-  const __nv_bfloat16* d = static_cast<const __nv_bfloat16*>(p.d_out) + x * DV;
   float acc = 0.f;
+  if (real) {
+    const uint4 o = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.out) + x * DV)[sub];
+    const uint4 d = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.d_out) + x * DV)[sub];
+    const uint32_t ow[4] = {o.x, o.y, o.z, o.w}, dw[4] = {d.x, d.y, d.z, d.w};
 #pragma unroll
-  for (int c = lane; c < DV; c += 32) acc += __bfloat162float(o[c]) * __bfloat162float(d[c]);
-#pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-  if (lane == 0) {
-    p.nd[row] = -acc;
-    p.nl2[row] = -p.lse[x] * 1.4426950408889634f;
+    for (int e = 0; e < 4; ++e) acc += bf16lo(ow[e]) * bf16lo(dw[e]) + bf16hi(ow[e]) * bf16hi(dw[e]);
   }
 #pragma unroll
-  for (int c = lane; c < R; c += 32) p.dq[x * R + c] = 0.f;
+  for (int off = TPR / 2; off >= 1; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+  if (!in_grid) return;
+  if (sub == 0) {
+    p.nd[row] = real ? -acc : 0.f;
+    p.nl2[row] = real ? -p.lse[x] * 1.4426950408889634f : -INFINITY;
+  }
+  if (!real) return;
+  float4* dq = reinterpret_cast<float4*>(p.dq + x * R);
+#pragma unroll
+  for (int c = sub; c < R / 4; c += TPR) dq[c] = make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
 // ---------------------------------------------------------------- main kernel
@@ -378,9 +384,10 @@ __global__ void __launch_bounds__(kBwdThreads, 1) bwd_main(const BackwardParams 
 template <int R, int DV>
 cudaError_t launch_t(const BackwardParams& p, cudaStream_t s, int* uns) {
   const long long rows = static_cast<long long>(p.B) * p.Hq * p.S_pad;
-  const long long pblocks = (rows + 7) / 8;
+  constexpr int rpb = kPrepThreads / (DV / 8);
+  const long long pblocks = (rows + rpb - 1) / rpb;
   if (pblocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-  bwd_prep<R, DV><<<static_cast<unsigned>(pblocks), 256, 0, s>>>(p);
+  bwd_prep<R, DV><<<static_cast<unsigned>(pblocks), kPrepThreads, 0, s>>>(p);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if constexpr (R <= 64) {
