@@ -365,6 +365,70 @@ __device__ void merge_segments(const DecodeParams& p, const float* merge, uint64
 struct DecodeMaps {
   CUtensorMap k, v;
 };
+// L2 prefetch of a CTA's first chunks, issued by its producer warp before the
+// dependent-launch wait: while the previous kernel on the stream finishes,
+// the CTA's first TMA reads after the wait then come from L2.  The context
+// lengths and page table read here may be stale (the previous kernel may
+// still write them); they are clamped so that every prefetched address lies
+// inside the cache, and a wrong guess only wastes the prefetch (L2 is
+// coherent, so nothing stale is ever read).  Batches of up to 32 sequences.
+template <int RB, int DV>
+__device__ void prefetch_first_chunks(const DecodeParams& p, int lane, int limit, int nunits) {
+  const int B = p.B, Hkv = p.Hkv;
+  int L = 0;
+  if (lane < B) {
+    L = p.seq_lens[lane];
+    if (p.fuse_append && L >= 0) ++L;
+    L = min(max(L, 0), limit);
+  }
+  const long long x = static_cast<long long>((L + kChunk - 1) / kChunk) * Hkv;  // units of sequence `lane`
+  long long inc = x;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const long long y = __shfl_up_sync(0xffffffffu, inc, off);
+    if (lane >= off) inc += y;
+  }
+  const long long T = __shfl_sync(0xffffffffu, inc, 31);
+  const long long pre = inc - x;
+  const int N = static_cast<int>(min(static_cast<long long>(gridDim.x), max((T + 3) / 4, 1LL)));
+  const int c = blockIdx.x;
+  if (T == 0 || c >= N) return;  // warp-uniform
+  const long long u_begin = T * c / N, u_end = T * (c + 1) / N;
+  const long long u = u_begin + lane;
+  int b = 0;
+  for (int bb = 0; bb < B; ++bb) {
+    const long long pb = __shfl_sync(0xffffffffu, pre, bb), xb = __shfl_sync(0xffffffffu, x, bb);
+    if (pb <= u && u < pb + xb) b = bb;
+  }
+  const int Lb = __shfl_sync(0xffffffffu, L, b);
+  const long long pb = __shfl_sync(0xffffffffu, pre, b);
+  const int nb = (Lb + kChunk - 1) / kChunk;
+  if (lane >= nunits || u >= u_end || nb == 0) return;
+  const long long off = u - pb;
+  const int g = static_cast<int>(off / nb), t0 = static_cast<int>(off % nb) * kChunk;
+  long long row;
+  int rows;
+  if (p.page_size == 0) {
+    row = (static_cast<long long>(b) * Hkv + g) * p.capacity + t0;
+    rows = min(kChunk, p.capacity - t0);
+  } else {
+    const int pidx = t0 >> p.page_shift;
+    if (pidx >= p.max_pages) return;
+    const int page = p.page_table[static_cast<long long>(b) * p.max_pages + pidx];
+    if (page < 0 || page >= p.num_pages) return;
+    const int in_page = t0 & (p.page_size - 1);
+    row = (static_cast<long long>(page) * Hkv + g) * p.page_size + in_page;
+    rows = min(kChunk, p.page_size - in_page);
+  }
+  if (rows <= 0) return;
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const unsigned char*>(p.k) + row * RB),
+               "r"(static_cast<uint32_t>(rows * RB))
+               : "memory");
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(static_cast<const unsigned char*>(p.v) + row * DV * 2),
+               "r"(static_cast<uint32_t>(rows * DV * 2))
+               : "memory");
+}
+
 
 template <int R, int DV, int G, int KF>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -397,14 +461,15 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
     }
     fence_barrier_init();
   }
-  // everything above touches only shared memory and parameters
-  pdl_wait();
-  pdl_trigger();
-
   // ---- clamped context lengths and prefix sums of units
   int limit = p.max_seq_len;
   if (p.page_size == 0) limit = min(limit, p.capacity);
   else limit = min(limit, p.max_pages * p.page_size);
+  // before the wait only reads that may be stale and L2 prefetches are issued
+  if (warp == kCW && B <= 32) prefetch_first_chunks<C::RB, DV>(p, lane, limit, C::NSTAGE);
+  pdl_wait();
+  pdl_trigger();
+
   for (int b = tid; b < B; b += kThreads) {
     int L = p.seq_lens[b];
     if (p.fuse_append && L >= 0) ++L;  // the appended token is part of the context
