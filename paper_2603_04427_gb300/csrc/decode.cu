@@ -372,6 +372,8 @@ struct DecodeMaps {
 // still write them); they are clamped so that every prefetched address lies
 // inside the cache, and a wrong guess only wastes the prefetch (L2 is
 // coherent, so nothing stale is ever read).  Batches of up to 32 sequences.
+// Twice the ring depth measured best on the Mistral GQA shape (28.5 us
+// against 29.2 us for one ring, 29.2 us for four).
 template <int RB, int DV>
 __device__ void prefetch_first_chunks(const DecodeParams& p, int lane, int limit, int nunits) {
   const int B = p.B, Hkv = p.Hkv;
@@ -466,7 +468,7 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
   if (p.page_size == 0) limit = min(limit, p.capacity);
   else limit = min(limit, p.max_pages * p.page_size);
   // before the wait only reads that may be stale and L2 prefetches are issued
-  if (warp == kCW && B <= 32) prefetch_first_chunks<C::RB, DV>(p, lane, limit, C::NSTAGE);
+  if (warp == kCW && B <= 32) prefetch_first_chunks<C::RB, DV>(p, lane, limit, 2 * C::NSTAGE);
   pdl_wait();
   pdl_trigger();
 
