@@ -228,7 +228,13 @@ size_t tk_decode_workspace_size(const tk_cache_desc* desc, int32_t max_seq_len);
  *              (0 gives a zero output row)
  *   max_seq_len: host upper bound of seq_lens, sizes the launch; a larger
  *              device value is clamped to it and flagged.
- *   out      : device [batch][h_q][d_v], TK_F32 or TK_BF16
+ *   out      : [batch][h_q][d_v], TK_F32 or TK_BF16: device memory, or
+ *              page-locked host memory (cudaHostAlloc / cudaHostRegister):
+ *              under unified addressing the kernel then stores the rows
+ *              straight into host memory (zero-copy), which replaces a
+ *              separate device-to-host copy when the result is wanted on the
+ *              host.  Like every pointer here it is not validated: any other
+ *              memory faults like an invalid device pointer.
  *   scale    : multiplies q.k (for int8 keys, q.(code * k_scale))
  *   workspace: device scratch of tk_decode_workspace_size bytes, aligned to
  *              256 bytes (see tk_decode_workspace_size).
@@ -267,6 +273,14 @@ tk_status tk_attn_decode_append(const tk_cache_desc* desc, const void* q, void* 
                                 const int32_t* seq_lens, const void* k_new, const void* v_new,
                                 int32_t max_seq_len, void* out, int32_t out_dtype, float scale,
                                 void* workspace, size_t workspace_bytes, void* stream);
+
+/* Stream-ordered copy of `bytes` bytes between any two of device memory and
+ * page-locked host memory (cudaMemcpyAsync with the direction taken from the
+ * pointers), for serving loops that bring a step's inputs from the host:
+ * issued natively, it costs the step less host time than a copy through a
+ * framework.  bytes == 0 is a no-op; NULL pointers give TK_ERR_INVALID_ARG,
+ * a failed enqueue TK_ERR_CUDA.  Not part of the paper's method.            */
+tk_status tk_copy_async(void* dst, const void* src, size_t bytes, void* stream);
 
 /* Size of the fixed device scratch array used by tk_attn_decode_noalloc. */
 #define TK_DECODE_NOALLOC_SCRATCH_BYTES (8u << 20)

@@ -23,8 +23,8 @@ LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtk.so")
 
 EXPORTED = ("tk_kv_append", "tk_attn_prefill", "tk_decode_workspace_size", "tk_attn_decode",
             "tk_attn_decode_append", "tk_attn_decode_noalloc", "tk_attn_prefill_cached",
-            "tk_attn_forward", "tk_backward_workspace_size", "tk_attn_backward", "tk_get_device_error", "tk_status_string", "tk_last_error",
-            "tk_abi_version")
+            "tk_attn_forward", "tk_backward_workspace_size", "tk_attn_backward", "tk_copy_async",
+            "tk_get_device_error", "tk_status_string", "tk_last_error", "tk_abi_version")
 
 
 class TkError(RuntimeError):
@@ -69,6 +69,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
                                         sz, vp]),
         "tk_attn_decode_noalloc": (i32, [dp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp]),
         "tk_get_device_error": (i32, [ctypes.POINTER(i32), vp]),
+        "tk_copy_async": (i32, [vp, vp, sz, vp]),
         "tk_status_string": (ctypes.c_char_p, [i32]),
         "tk_last_error": (ctypes.c_char_p, []),
         "tk_abi_version": (i32, []),
@@ -98,6 +99,17 @@ def _ptr(t):
 def _stream(stream):
     s = torch.cuda.current_stream() if stream is None else stream
     return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need_out(t, name, device):
+    """An output: float32 or bfloat16, contiguous, on `device` or in page-locked host memory
+    (the kernel then writes it zero-copy)."""
+    if t.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError(f"{name} must be float32 or bfloat16")
+    if t.is_cuda:
+        _need(t, t.dtype, name, device)
+    elif not t.is_pinned() or not t.is_contiguous():
+        raise ValueError(f"{name} must be a CUDA tensor or a contiguous page-locked host tensor")
 
 
 def _need(t, dtype, name, device=None):
@@ -229,9 +241,7 @@ def tk_attn_decode_append(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_se
     _need(v_new, torch.bfloat16, "v_new", dev)
     _need(seq_lens, torch.int32, "seq_lens", dev)
     _need(workspace, torch.uint8, "workspace", dev)
-    if out.dtype not in (torch.float32, torch.bfloat16):
-        raise TypeError("out must be float32 or bfloat16")
-    _need(out, out.dtype, "out", dev)
+    _need_out(out, "out", dev)
     if tuple(q.shape) != (d.batch, d.h_q, d.r) or tuple(out.shape) != (d.batch, d.h_q, d.d_v):
         raise ValueError(f"q {tuple(q.shape)} / out {tuple(out.shape)} do not match the cache")
     if tuple(k_new.shape) != (d.batch, d.h_kv, d.r) or tuple(v_new.shape) != (d.batch, d.h_kv, d.d_v):
@@ -328,36 +338,65 @@ def tk_attn_prefill_cached(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_s
 
 
 class PreparedCall:
-    """One entry-point call with its arguments checked and marshalled once.
+    """Entry-point calls with their arguments checked and marshalled once.
 
     For serving loops whose buffers stay fixed between steps: calling the
-    object re-issues the same C call (same pointers, same stream) without the
-    per-call Python checks, and raises TkError on a non-OK status."""
+    object re-issues the same C calls in order (same pointers, same stream)
+    without the per-call Python checks, and raises TkError on a non-OK status."""
 
-    def __init__(self, name: str, args: tuple, keep: tuple):
-        self._fn = getattr(load_library(), name)
-        self._name = name
-        self._args = args
+    def __init__(self, name: str, args: tuple, keep: tuple, before: tuple = ()):
+        L = load_library()
+        self._calls = tuple((getattr(L, n), n, a) for n, a in (*before, (name, args)))
         self._keep = keep  # the tensors whose pointers are in args stay alive
 
     def __call__(self):
-        st = self._fn(*self._args)
-        if st != TK_OK:
-            _check(st, self._name)
+        for fn, name, args in self._calls:
+            st = fn(*args)
+            if st != TK_OK:
+                _check(st, name)
+
+
+def tk_copy_async(dst, src, stream=None):
+    """Stream-ordered copy between device memory and page-locked host memory (same byte size)."""
+    for t, n in ((dst, "dst"), (src, "src")):
+        if not t.is_contiguous() or not (t.is_cuda or t.is_pinned()):
+            raise ValueError(f"{n} must be contiguous, on a GPU or page-locked")
+    nb = dst.numel() * dst.element_size()
+    if src.numel() * src.element_size() != nb:
+        raise ValueError("dst and src differ in size")
+    _check(load_library().tk_copy_async(_ptr(dst), _ptr(src), nb, _stream(stream)), "tk_copy_async")
+    return dst
 
 
 def prepare_decode_append(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_seq_len: int, out,
-                          workspace, scale: float | None = None, stream=None) -> PreparedCall:
-    """tk_attn_decode_append with every argument checked once (see that function)."""
+                          workspace, scale: float | None = None, stream=None,
+                          copy_in=None) -> PreparedCall:
+    """tk_attn_decode_append with every argument checked once (see that function).
+
+    copy_in = (dst, src): a device tensor and a page-locked host tensor of the
+    same byte size, copied (tk_copy_async) before each decode -- e.g. the
+    step's q, k_new and v_new packed in one host buffer.  `out` may be a
+    page-locked host tensor: the kernel then writes the result there directly."""
     d = cache.desc
     dev = cache.k.device
     for t, n in ((q, "q"), (k_new, "k_new"), (v_new, "v_new")):
         _need(t, torch.bfloat16, n, dev)
     _need(seq_lens, torch.int32, "seq_lens", dev)
     _need(workspace, torch.uint8, "workspace", dev)
-    if out.dtype not in (torch.float32, torch.bfloat16):
-        raise TypeError("out must be float32 or bfloat16")
-    _need(out, out.dtype, "out", dev)
+    _need_out(out, "out", dev)
+    before = ()
+    keep_in = ()
+    if copy_in is not None:
+        dst, src = copy_in
+        if not dst.is_cuda or dst.device != dev or not dst.is_contiguous():
+            raise ValueError("copy_in: dst must be a contiguous tensor on the cache's device")
+        if src.is_cuda or not src.is_pinned() or not src.is_contiguous():
+            raise ValueError("copy_in: src must be a contiguous page-locked host tensor")
+        nb = dst.numel() * dst.element_size()
+        if src.numel() * src.element_size() != nb:
+            raise ValueError("copy_in: dst and src differ in size")
+        before = (("tk_copy_async", (_ptr(dst), _ptr(src), ctypes.c_size_t(nb), _stream(stream))),)
+        keep_in = (dst, src)
     if tuple(q.shape) != (d.batch, d.h_q, d.r) or tuple(out.shape) != (d.batch, d.h_q, d.d_v):
         raise ValueError(f"q {tuple(q.shape)} / out {tuple(out.shape)} do not match the cache")
     if tuple(k_new.shape) != (d.batch, d.h_kv, d.r) or tuple(v_new.shape) != (d.batch, d.h_kv, d.d_v):
@@ -368,7 +407,7 @@ def prepare_decode_append(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_se
             _ptr(out), TK_F32 if out.dtype == torch.float32 else TK_BF16, ctypes.c_float(scale),
             _ptr(workspace), ctypes.c_size_t(workspace.numel()), _stream(stream))
     return PreparedCall("tk_attn_decode_append", args,
-                        (cache, q, k_new, v_new, seq_lens, out, workspace))
+                        (cache, q, k_new, v_new, seq_lens, out, workspace) + keep_in, before)
 
 
 def tk_attn_prefill(q, k, v, out, scale: float | None = None, causal: bool = True, stream=None):

@@ -408,6 +408,14 @@ tk_status tk_attn_decode_append(const tk_cache_desc* desc, const void* q, void* 
                      max_seq_len, out, out_dtype, scale, workspace, workspace_bytes, stream);
 }
 
+tk_status tk_copy_async(void* dst, const void* src, size_t bytes, void* stream) {
+  if (bytes == 0) return TK_OK;
+  if (!dst || !src) return fail(TK_ERR_INVALID_ARG, "copy: NULL pointer");
+  const cudaError_t e = cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDefault, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync");
+  return TK_OK;
+}
+
 tk_status tk_get_device_error(int32_t* code_out, void* stream) {
   if (!code_out) return fail(TK_ERR_INVALID_ARG, "code_out is NULL");
   DeviceInfo* dev;

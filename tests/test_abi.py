@@ -168,3 +168,19 @@ def test_prefill_validation(lib):
     assert P(FAKE, FAKE, FAKE, FAKE, tb.TK_BF16, 2, 4, 4, -1, 32, 128, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG
     assert P(None, None, None, None, tb.TK_BF16, 2, 4, 4, 0, 32, 128, 0.1, 1, None) == tb.TK_OK
     assert P(None, FAKE, FAKE, FAKE, tb.TK_BF16, 2, 4, 4, 64, 32, 128, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG
+
+
+def test_copy_async_validation(lib):
+    """tk_copy_async: an empty copy is a no-op and NULL pointers are rejected, before any CUDA call."""
+    assert lib.tk_copy_async(None, None, 0, None) == tb.TK_OK
+    assert lib.tk_copy_async(None, FAKE, 16, None) == tb.TK_ERR_INVALID_ARG
+    assert lib.tk_copy_async(FAKE, None, 16, None) == tb.TK_ERR_INVALID_ARG
+
+
+def test_host_output_needs_page_locked_memory():
+    """The binding accepts a host output only when it is page-locked (the kernel writes it zero-copy)."""
+    import torch
+    with pytest.raises(ValueError):
+        tb._need_out(torch.empty(4, 8), "out", None)          # pageable host memory
+    with pytest.raises(TypeError):
+        tb._need_out(torch.empty(4, 8, dtype=torch.float16), "out", None)

@@ -199,3 +199,38 @@ def test_prepared_call_equals_direct_call():
     with pytest.raises(ValueError):
         tb.prepare_decode_append(cache, q[:, :4], k1, v1, sl, 641, out_p,
                                  tb.decode_workspace(cache.desc, 641))
+
+
+def test_prepared_call_with_host_input_and_zero_copy_output():
+    """copy_in from page-locked host memory and a page-locked host `out` (written by the
+    kernel directly) give the same bits as the all-device call."""
+    require_gpu()
+    B, hq, hkv, r, dv = 4, 32, 8, 32, 128
+    lens = [100, 640, 1, 300]
+    cache, _, _ = _make(B, hq, hkv, r, dv, lens, False, 0, seed=61)
+    other = _clone(cache)
+    q = inputs.normal_bf16((B, hq, r), seed=62, device="cuda")
+    k1 = inputs.normal_bf16((B, hkv, r), seed=63, device="cuda")
+    v1 = inputs.normal_bf16((B, hkv, dv), seed=64, device="cuda")
+    sl = torch.tensor(lens, dtype=torch.int32, device="cuda")
+    out_d = torch.empty(B, hq, dv, device="cuda")
+    tb.tk_attn_decode_append(other, q, k1, v1, sl, 641, out_d, tb.decode_workspace(other.desc, 641))
+    # the step's q, k_new, v_new packed in one device buffer, filled from one host buffer
+    io = torch.empty(q.numel() + k1.numel() + v1.numel(), dtype=torch.bfloat16, device="cuda")
+    hio = torch.cat([q.flatten(), k1.flatten(), v1.flatten()]).cpu().pin_memory()
+    nq, nk = q.numel(), k1.numel()
+    qv = io[:nq].view(B, hq, r)
+    kv = io[nq:nq + nk].view(B, hkv, r)
+    vv = io[nq + nk:].view(B, hkv, dv)
+    out_h = torch.full((B, hq, dv), float("nan")).pin_memory()
+    stream = torch.cuda.Stream()
+    call = tb.prepare_decode_append(cache, qv, kv, vv, sl, 641, out_h, tb.decode_workspace(cache.desc, 641),
+                                    stream=stream, copy_in=(io, hio))
+    call()
+    stream.synchronize()
+    assert tb.tk_get_device_error() == 0
+    assert torch.equal(out_h, out_d.cpu())
+    _same_cache(other, cache)
+    with pytest.raises(ValueError):
+        tb.prepare_decode_append(cache, qv, kv, vv, sl, 641, out_h, tb.decode_workspace(cache.desc, 641),
+                                 copy_in=(io, hio[:-1]))
