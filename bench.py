@@ -507,6 +507,17 @@ def run_reference(args, rank):
     print(json.dumps(line), flush=True)
 
 
+def max_over_ranks(dist, values, device):
+    """Element-wise maximum of `values` over all ranks (the slowest rank's times);
+    `values` unchanged on a single process (dist None)."""
+    if dist is None:
+        return [float(x) for x in values]
+    import torch
+    t = torch.tensor([float(x) for x in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t]
+
+
 # ----------------------------------------------------------------------------- main
 
 def main():
@@ -575,17 +586,11 @@ def main():
     sec_dec = measure_decode(rig, args.steps, args.warmup, mode="decode")
     torch.cuda.synchronize()
     clk = clocks.stop()
-    if dist:
-        t = torch.tensor([sec_step, sec_dec, sec_two], dtype=torch.float64, device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        sec_step, sec_dec, sec_two = float(t[0]), float(t[1]), float(t[2])
+    sec_step, sec_dec, sec_two = max_over_ranks(dist, (sec_step, sec_dec, sec_two), device)
     n = world
     value = n * rig.kv_bytes / sec_step / 1e9
     e2e_dt, h2d, d2h = measure_decode_e2e(rig, min(args.steps, 5000))
-    if dist:
-        t = torch.tensor([e2e_dt], dtype=torch.float64, device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_dt = float(t[0])
+    (e2e_dt,) = max_over_ranks(dist, (e2e_dt,), device)
     achieved = (rig.kv_bytes + rig.io_bytes) / sec_dec / 1e9
     dec_hash = source_hash("decode.cu", "common.cuh")
     line = {
