@@ -176,8 +176,8 @@ size_t tk_backward_workspace_size(int32_t batch, int32_t h_q, int32_t seq);
  *   workspace: tk_backward_workspace_size bytes, 256-byte aligned (scratch)
  *   scale, causal: as in the forward.
  * The products run on the tensor cores with bf16 operands (P and dS rounded
- * to bf16) and fp32 accumulation (tcgen05 for r <= 64, mma.sync for
- * r = 128); dq is accumulated across key tiles with fp32 reduce-adds, so its
+ * to bf16) and fp32 accumulation (tcgen05, accumulators in tensor memory);
+ * dq is accumulated across key tiles with fp32 reduce-adds, so its
  * low bits may vary run to run.  Two launches (preprocessing, gradients).    */
 tk_status tk_attn_backward(const void* q, const void* k, const void* v, const void* out,
                            const void* d_out, const float* lse, float* dq, float* dk, float* dv,

@@ -1,6 +1,6 @@
-// Gradient kernel of thin-key attention on the 5th-generation tensor cores
-// (r <= 64): tcgen05.mma with accumulators in tensor memory, operands staged
-// in shared memory by TMA.
+// Gradient kernel of thin-key attention on the 5th-generation tensor cores:
+// tcgen05.mma with accumulators in tensor memory, operands staged in shared
+// memory by TMA.
 //
 // Paper: Section 2.1, Eqs. 1-4 (the forward being differentiated); training
 // with thin keys is Sections 3.2-3.3.  Per head, with p = softmax(scale q k^T)
@@ -43,6 +43,9 @@
 // TMEM columns: [0,64) S^T_0, [64,128) dP^T_0, [128,192) S^T_1,
 // [192,256) dP^T_1, then dV (d_v), dK (r), dQ (r), and where they fit P^T_0,
 // P^T_1 (32 columns each; otherwise P^T_h sits in the first 32 of S^T_h).
+// At r = 128, dV, dK and dQ do not fit beside the score tiles: dQ_i is then
+// computed over S^T_1 / dP^T_1 once the half-1 softmax has consumed them,
+// warps 4-7 read it back at once, and the next half-1 scores follow.
 #include <algorithm>
 #include <type_traits>
 
@@ -64,34 +67,45 @@ constexpr int align1k(int x) { return (x + 1023) / 1024 * 1024; }
 
 template <int R, int DV>
 struct TCfg {
-  static_assert(R <= 64, "thin keys only: the r = 128 backward runs on mma.sync");
-  // Q / K rows are r bf16 = 2r bytes, one swizzle span (32, 64 or 128 bytes)
-  static constexpr int QK_SW = 2 * R;
+  // Q / K rows are r bf16 = 2r bytes: one swizzle span of min(2r, 128) bytes,
+  // in QK_NBOX boxes of QK_BOXW columns (two 128-byte boxes at r = 128)
+  static constexpr int QK_SW = 2 * R < 128 ? 2 * R : 128;
+  static constexpr int QK_NBOX = 2 * R / QK_SW;
+  static constexpr int QK_BOXW = QK_SW / 2;
   static constexpr uint32_t QK_LAYOUT = QK_SW == 32 ? 6u : (QK_SW == 64 ? 4u : 2u);
-  static constexpr int KB = kKeys * R * 2;         // K tile
-  static constexpr int VB = kKeys * DV * 2;        // V tile (DV / 64 boxes)
-  // Q / dO arrive in 64-query half tiles, a ring of 4 slots: a slot is
+  static constexpr int KSTEP_PER_BOX = QK_SW / 32;  // 16-column K steps per box
+  static constexpr int KBOX = kKeys * QK_SW;        // one box of the K tile
+  static constexpr int KB = QK_NBOX * KBOX;         // K tile
+  static constexpr int VB = kKeys * DV * 2;         // V tile (DV / 64 boxes)
+  // Q / dO arrive in 64-query half tiles through a ring of slots: a slot is
   // released as soon as its half's dV / dK products have read it
-  static constexpr int QHB = kHalfQ * R * 2;       // Q half tile (one box)
-  static constexpr int OHB = kHalfQ * DV * 2;      // dO half tile (DV / 64 boxes)
-  static constexpr int OBOX = kHalfQ * 128;        // one 64-column box of a half tile
+  static constexpr int QHBOX = kHalfQ * QK_SW;      // one box of a Q half tile
+  static constexpr int QHB = QK_NBOX * QHBOX;       // Q half tile
+  static constexpr int OHB = kHalfQ * DV * 2;       // dO half tile (DV / 64 boxes)
+  static constexpr int OBOX = kHalfQ * 128;         // one 64-column box of a dO half tile
   static constexpr int SL_Q = 0, SL_O = align1k(QHB), SL_L = SL_O + OHB, SL_D = SL_L + kHalfQ * 4;
   static constexpr int SLOT = align1k(SL_D + kHalfQ * 4);
-  static constexpr int DSB = kKeys * kQT * 2;      // dS^T tile: [2 halves][128 keys][64 queries]
-  // dQ tile staged for the TMA reduce-add: softmax warpgroup h stages columns
-  // [h R/2, (h+1) R/2), each warp its 32 rows as one box swizzled over
-  // DQ_SW = 2r bytes (conflict-free row-per-thread stores)
-  static constexpr int DQ_W = R / 2;
+  static constexpr int DSB = kKeys * kQT * 2;       // dS^T tile: [2 halves][128 keys][64 queries]
+  // dQ of a tile in TMEM: in columns of its own where they fit (r <= 64), else
+  // over S^T_1 / dP^T_1 once the half-1 softmax has consumed them (r = 128)
+  static constexpr bool DQ_OWN = 256 + DV + 2 * R <= kTmemColsTc;
+  // dQ read back and staged for the TMA reduce-add, boxes of DQ_W fp32
+  // columns x 32 rows (one per warp) swizzled over DQ_SW bytes: with its own
+  // columns each softmax warpgroup takes R / 2 columns after the next tile's
+  // softmax; over S^T_1 / dP^T_1, warps 4-7 take all R at once, right after
+  // their softmax, and stage them 32 columns at a time
+  static constexpr int DQ_W = DQ_OWN ? R / 2 : 32;
   static constexpr int DQ_SW = DQ_W * 4;
   static constexpr int DQ_LAYOUT_SHIFT = DQ_SW == 128 ? 0 : (DQ_SW == 64 ? 1 : 2);
-  static constexpr int DQB = kQT * R * 4;
+  static constexpr int DQB = DQ_OWN ? kQT * R * 4 : 4 * 32 * DQ_SW;
   static constexpr int OFF_K = 0;
   static constexpr int OFF_V = align1k(KB);
   static constexpr int OFF_SL = OFF_V + VB;
-  static constexpr int NSLOT = 4;   // half-tile slots (a fifth, where it fits, measured slower)
-  // without the dS tiles: K, V, the ring, the dQ stage, barriers, alignment slack
-  static constexpr int FIXED = OFF_SL + NSLOT * SLOT + DQB + 256 + 1024;
-  static constexpr int NDS = FIXED + 2 * DSB <= 227 * 1024 ? 2 : 1;   // dS^T tiles in flight
+  // without the dS tiles: K, V, a ring of n slots, the dQ stage, barriers, alignment slack
+  static constexpr int fixed(int n) { return OFF_SL + n * SLOT + DQB + 256 + 1024; }
+  static constexpr int NDS = fixed(4) + 2 * DSB <= 227 * 1024 ? 2 : 1;   // dS^T tiles in flight
+  // half-tile slots: 4 (a fifth, where it fits, measured slower), 3 where 4 do not fit
+  static constexpr int NSLOT = fixed(4) + NDS * DSB <= 227 * 1024 ? 4 : 3;
   static constexpr int OFF_DS = OFF_SL + NSLOT * SLOT;
   static constexpr int OFF_DQ = OFF_DS + NDS * DSB;
   static constexpr int OFF_BAR = OFF_DQ + DQB;
@@ -101,9 +115,9 @@ struct TCfg {
   // TMEM columns
   static constexpr int T_S = 0;          // + 128 h: S^T_h
   static constexpr int T_DP = 64;        // + 128 h: dP^T_h
-  static constexpr int T_DV = 256, T_DK = 256 + DV, T_DQ = 256 + DV + R;
-  static_assert(T_DQ + R <= kTmemColsTc, "TMEM columns");
-  static constexpr bool P_OWN = T_DQ + R + 2 * (kHalfQ / 2) <= kTmemColsTc;  // P^T in columns of its own
+  static constexpr int T_DV = 256, T_DK = 256 + DV, T_DQ = DQ_OWN ? 256 + DV + R : 128;
+  static_assert(T_DK + R <= kTmemColsTc && (!DQ_OWN || T_DQ + R <= kTmemColsTc), "TMEM columns");
+  static constexpr bool P_OWN = DQ_OWN && T_DQ + R + 2 * (kHalfQ / 2) <= kTmemColsTc;  // P^T in columns of its own
   static constexpr int T_P = P_OWN ? T_DQ + R : T_S;   // + (P_OWN ? 32 : 128) h: P^T_h
   static constexpr int P_STRIDE = P_OWN ? kHalfQ / 2 : 128;
   // With P^T in its own columns and two dS tiles, the next tile's scores of a
@@ -249,7 +263,7 @@ bwd_tc_kernel(const __grid_constant__ TcMaps maps, const BackwardParams p) {
     }
     for (int s = 0; s < NDS; ++s) mbar_init(&ds_free[s], 1);
     mbar_init(dq_full, 1);
-    mbar_init(dq_empty, 256);
+    mbar_init(dq_empty, C::DQ_OWN ? 256 : 128);
     mbar_init(acc_full, 1);
     fence_barrier_init();
   }
@@ -270,7 +284,8 @@ bwd_tc_kernel(const __grid_constant__ TcMaps maps, const BackwardParams p) {
       prefetch_map(&maps.v);
       prefetch_map(&maps.d_out);
       mbar_arrive_expect_tx(kv_full, C::KB + C::VB);
-      tma_load_3d(smem + C::OFF_K, &maps.k, 0, j * kKeys, kv_plane, kv_full);
+      for (int x = 0; x < C::QK_NBOX; ++x)
+        tma_load_3d(smem + C::OFF_K + x * C::KBOX, &maps.k, x * C::QK_BOXW, j * kKeys, kv_plane, kv_full);
       for (int x = 0; x < DV / 64; ++x)
         tma_load_3d(smem + C::OFF_V + x * kBoxB, &maps.v, 64 * x, j * kKeys, kv_plane, kv_full);
       int issued = 0;
@@ -281,7 +296,8 @@ bwd_tc_kernel(const __grid_constant__ TcMaps maps, const BackwardParams p) {
         const int bh = b * p.Hq + tile_head(t), row = tile_q(t) * kQT + h * kHalfQ;
         unsigned char* sb = smem + C::OFF_SL + sl * C::SLOT;
         mbar_arrive_expect_tx(&sl_full[sl], C::QHB + C::OHB + 2 * kHalfQ * 4);
-        tma_load_3d(sb + C::SL_Q, &maps.q, 0, row, bh, &sl_full[sl]);
+        for (int x = 0; x < C::QK_NBOX; ++x)
+          tma_load_3d(sb + C::SL_Q + x * C::QHBOX, &maps.q, x * C::QK_BOXW, row, bh, &sl_full[sl]);
         for (int x = 0; x < DV / 64; ++x)
           tma_load_3d(sb + C::SL_O + x * C::OBOX, &maps.d_out, 64 * x, row, bh, &sl_full[sl]);
         const size_t srow = static_cast<size_t>(bh) * p.S_pad + row;
@@ -300,9 +316,9 @@ bwd_tc_kernel(const __grid_constant__ TcMaps maps, const BackwardParams p) {
     const uint32_t s_base = smem_addr(smem);
     // one descriptor serves a tile read K-major and MN-major: SBO is the stride of
     // 8-row groups either way, LBO the stride of MN atoms (unused when N fits one)
-    const Desc dK_d = make_desc(s_base + C::OFF_K, 16, 8 * C::QK_SW, C::QK_LAYOUT);       // K
+    const Desc dK_d = make_desc(s_base + C::OFF_K, C::KBOX, 8 * C::QK_SW, C::QK_LAYOUT);  // K
     const Desc dV_a = make_desc(s_base + C::OFF_V, 16, 1024, 2u);                         // V, K-major
-    const Desc dQ_b = make_desc(s_base + C::OFF_SL + C::SL_Q, 16, 8 * C::QK_SW, C::QK_LAYOUT);  // Q_h
+    const Desc dQ_b = make_desc(s_base + C::OFF_SL + C::SL_Q, C::QHBOX, 8 * C::QK_SW, C::QK_LAYOUT);  // Q_h
     const Desc dO_bk = make_desc(s_base + C::OFF_SL + C::SL_O, 16, 1024, 2u);             // dO_h, K-major
     const Desc dO_bm = make_desc(s_base + C::OFF_SL + C::SL_O, C::OBOX, 1024, 2u);        // dO_h, MN-major
     const Desc dS_ak = make_desc(s_base + C::OFF_DS, 16, 1024, 2u);                       // dS^T, K-major
@@ -310,8 +326,11 @@ bwd_tc_kernel(const __grid_constant__ TcMaps maps, const BackwardParams p) {
     auto issue_sdp = [&](int t, int h) {   // S^T_h, dP^T_h of tile t
       const uint32_t so = slot_of(t, h) * C::SLOT;
 #pragma unroll
-      for (int k = 0; k < R / 16; ++k)
-        mma_ss_e(tmem + C::T_S + 128 * h, dK_d.at(k * 32), dQ_b.at(so + k * 32), C::ID_S, k > 0);
+      for (int k = 0; k < R / 16; ++k) {
+        const uint32_t kb = (k / C::KSTEP_PER_BOX), ko = (k % C::KSTEP_PER_BOX) * 32;
+        mma_ss_e(tmem + C::T_S + 128 * h, dK_d.at(kb * C::KBOX + ko), dQ_b.at(so + kb * C::QHBOX + ko), C::ID_S,
+                 k > 0);
+      }
 #pragma unroll
       for (int k = 0; k < DV / 16; ++k)
         mma_ss_e(tmem + C::T_DP + 128 * h, dV_a.at((k / 4) * kBoxB + (k % 4) * 32),
@@ -391,10 +410,15 @@ bwd_tc_kernel(const __grid_constant__ TcMaps maps, const BackwardParams p) {
           issue_dvdk(t, h);
           if (h == 1) {
             // dQ before the next tile's half-1 scores: with one dS tile the next
-            // tile's half-0 dS waits for it
-            if (t > 0 && !(ok = wait_all(dq_empty, (t - 1) & 1))) break;
+            // tile's half-0 dS waits for it, and without columns of its own dQ
+            // occupies S^T_1 / dP^T_1 until warps 4-7 have read it
+            if (C::DQ_OWN && t > 0 && !(ok = wait_all(dq_empty, (t - 1) & 1))) break;
             tc_fence_after();
             issue_dq(t);
+            if (!C::DQ_OWN && next) {
+              if (!(ok = wait_all(dq_empty, t & 1))) break;
+              tc_fence_after();
+            }
           }
           if (!C::P_OWN && next) issue_sdp(t + 1, h);
         }
@@ -416,7 +440,8 @@ bwd_tc_kernel(const __grid_constant__ TcMaps maps, const BackwardParams p) {
     // read from TMEM after the next tile's softmax (dq_fetch), then staged in
     // shared memory and added into global dq by a TMA reduce per warp (its 32
     // rows), so that no warp waits for another (dq_store).
-    unsigned char* dq_box = smem + C::OFF_DQ + h * (kQT * C::DQ_SW) + (warp & 3) * (32 * C::DQ_SW);
+    unsigned char* dq_box =
+        smem + C::OFF_DQ + (C::DQ_OWN ? h * (kQT * C::DQ_SW) : 0) + (warp & 3) * (32 * C::DQ_SW);
     uint32_t wq[C::DQ_W];
     bool dq_ok = false;
     auto dq_fetch = [&](int t) {
@@ -450,6 +475,50 @@ bwd_tc_kernel(const __grid_constant__ TcMaps maps, const BackwardParams p) {
       }
       if (!dq_ok) ok = false;
       dq_ok = false;
+    };
+    // r = 128 (dQ over S^T_1 / dP^T_1): warps 4-7 read dQ_t right after their
+    // softmax of tile t, 64 columns at a time (the first half staged before the
+    // second is read), which then releases S^T_1 / dP^T_1 for the next scores;
+    // each half is added into dq DQ_W columns at a time
+    auto dq_all = [&](int t) {
+      static_assert(C::DQ_OWN || R == 128, "dQ over S^T_1 / dP^T_1 is laid out for r = 128");
+      const bool okw = __all_sync(0xffffffffu, ok && mbar_wait(dq_full, t & 1, p.err));
+      const int row0 = tile_q(t) * kQT + (warp & 3) * 32;
+      if (okw) tc_fence_after();
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        uint32_t w[64];
+        if (okw) {
+          tmem_ld64(tmem + C::T_DQ + 64 * half + lane_off, w);
+          if (half == 1) {
+            tc_fence_before();
+            mbar_arrive(dq_empty);
+          }
+        }
+        if (okw && row0 < S) {
+#pragma unroll
+          for (int ps = 0; ps < 64 / C::DQ_W; ++ps) {
+            if (lane == 0 && pending) bulk_wait_read_all();   // the previous reduce has read the box
+            __syncwarp();
+#pragma unroll
+            for (int c = 0; c < C::DQ_SW / 16; ++c) {
+              const int pc = c ^ ((lane >> C::DQ_LAYOUT_SHIFT) & (C::DQ_SW / 16 - 1));
+              const int e = ps * C::DQ_W + 4 * c;
+              *reinterpret_cast<float4*>(dq_box + lane * C::DQ_SW + pc * 16) =
+                  make_float4(__uint_as_float(w[e]) * p.scale, __uint_as_float(w[e + 1]) * p.scale,
+                              __uint_as_float(w[e + 2]) * p.scale, __uint_as_float(w[e + 3]) * p.scale);
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              tma_reduce_add_3d(&maps.dq, dq_box, 64 * half + ps * C::DQ_W, row0, b * p.Hq + tile_head(t));
+              bulk_commit();
+              pending = true;
+            }
+          }
+        }
+      }
+      if (!okw) ok = false;
     };
     for (int t = 0; t < n_tiles; ++t) {
       const int sl = slot_of(t, h), buf = t % NDS;
@@ -515,12 +584,16 @@ bwd_tc_kernel(const __grid_constant__ TcMaps maps, const BackwardParams p) {
         tc_fence_before();
         mbar_arrive(&p_ready[h]);
       }
-      if (t > 0) {
-        dq_fetch(t - 1);
-        dq_store(t - 1);
+      if constexpr (C::DQ_OWN) {
+        if (t > 0) {
+          dq_fetch(t - 1);
+          dq_store(t - 1);
+        }
+      } else if (h == 1) {
+        dq_all(t);
       }
     }
-    if (n_tiles > 0) {
+    if (C::DQ_OWN && n_tiles > 0) {
       dq_fetch(n_tiles - 1);
       dq_store(n_tiles - 1);
     }
@@ -551,8 +624,8 @@ template <int R, int DV>
 cudaError_t launch_tc(const BackwardParams& p, cudaStream_t stream) {
   using C = TCfg<R, DV>;
   TcMaps maps;
-  if (!make_map(&maps.q, p.q, R, p.S, p.B * p.Hq, R, kHalfQ, C::QK_SW) ||
-      !make_map(&maps.k, p.k, R, p.S, p.B * p.Hkv, R, kKeys, C::QK_SW) ||
+  if (!make_map(&maps.q, p.q, R, p.S, p.B * p.Hq, C::QK_BOXW, kHalfQ, C::QK_SW) ||
+      !make_map(&maps.k, p.k, R, p.S, p.B * p.Hkv, C::QK_BOXW, kKeys, C::QK_SW) ||
       !make_map(&maps.v, p.v, DV, p.S, p.B * p.Hkv, 64, kKeys, 128) ||
       !make_map(&maps.d_out, p.d_out, DV, p.S, p.B * p.Hq, 64, kHalfQ, 128) ||
       !make_map(&maps.dq, p.dq, R, p.S, p.B * p.Hq, C::DQ_W, 32, C::DQ_SW, true))
@@ -584,6 +657,7 @@ cudaError_t launch_backward_tc(const BackwardParams& p, cudaStream_t stream, int
     case 16: return tc_by_dv<16>(p, stream, unsupported);
     case 32: return tc_by_dv<32>(p, stream, unsupported);
     case 64: return tc_by_dv<64>(p, stream, unsupported);
+    case 128: return tc_by_dv<128>(p, stream, unsupported);
   }
   *unsupported = 1;
   return cudaSuccess;

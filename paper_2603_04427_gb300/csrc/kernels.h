@@ -127,7 +127,7 @@ struct BackwardParams {
 inline int backward_rows(int S) { return (S + 127) / 128 * 128; }
 
 cudaError_t launch_backward(const BackwardParams& p, cudaStream_t stream, int* unsupported);
-// The tensor-memory gradient kernel (r <= 64), after the preprocessing pass.
+// The tensor-memory gradient kernel, after the preprocessing pass.
 cudaError_t launch_backward_tc(const BackwardParams& p, cudaStream_t stream, int* unsupported);
 
 cudaError_t launch_prefill(const PrefillParams& p, cudaStream_t stream, int* unsupported);
