@@ -454,6 +454,8 @@ f = lambda t: bf16_bits_to_f64(t.view(torch.int16).numpy())
 k = f(inputs.normal_bf16((1, n_groups, L, r), seed + 1))
 v = f(inputs.normal_bf16((1, n_groups, L, dv), seed + 2))
 q = f(inputs.normal_bf16((1, n_groups * G, r), seed + 3))
+print("ready", flush=True)   # inputs built; the timed work starts on the parent's word
+sys.stdin.readline()
 for _ in range(warm):
     oa.attention_decode(q, k, v, [L], 1.0 / r ** 0.5)
 t0 = time.perf_counter()
@@ -464,21 +466,51 @@ print(json.dumps({"sec": el, "reps": reps, "bytes": cm.decode_kv_bytes([L] * n_g
 """
 
 
-def cpu_oracle_decode(w, n_groups: int, reps: int, warmup: int = 1):
-    """Time `reps` oracle decodes of a sample of the workload on one host thread, in a fresh process."""
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_oracle_decode(w, n_groups: int, reps: int, warmup: int = 1, procs: int = 1):
+    """Time `reps` oracle decodes of a sample of the workload: `procs` fresh
+    single-threaded processes, each on its share of the n_groups (sequence, kv
+    head) groups, start their timed loops together; throughput = all their
+    bytes / the slowest one's time."""
+    procs = max(1, min(procs, n_groups))
+    shares = [n_groups // procs + (1 if k < n_groups % procs else 0) for k in range(procs)]
     env = dict(os.environ, TK_ROOT=ROOT, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1",
                MKL_NUM_THREADS="1", CUDA_VISIBLE_DEVICES="")
-    args = [str(x) for x in (w.batch, w.h_q, w.h_kv, w.r, w.d_v, w.seq, w.seed, n_groups, reps, warmup)]
-    out = subprocess.run([sys.executable, "-c", CPU_CHILD] + args, env=env, capture_output=True,
-                         text=True, timeout=900)
-    if out.returncode != 0:
-        raise RuntimeError(out.stderr[-2000:])
-    d = json.loads(out.stdout.strip().splitlines()[-1])
-    return {"value": d["bytes"] / d["sec"] / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
-            "sec": d["sec"], "reps": reps,
+    children = []
+    for k, share in enumerate(shares):
+        args = [str(x) for x in (w.batch, w.h_q, w.h_kv, w.r, w.d_v, w.seq, w.seed + 7 * k, share, reps, warmup)]
+        children.append(subprocess.Popen([sys.executable, "-c", CPU_CHILD] + args, env=env, text=True,
+                                         stdin=subprocess.PIPE, stdout=subprocess.PIPE,
+                                         stderr=subprocess.PIPE))
+    try:
+        for c in children:   # every child has built its inputs
+            if c.stdout.readline().strip() != "ready":
+                raise RuntimeError(c.stderr.read()[-2000:])
+        for c in children:
+            c.stdin.write("go\n")
+            c.stdin.flush()
+        outs = [c.communicate(timeout=900) for c in children]
+    finally:
+        for c in children:
+            if c.poll() is None:
+                c.kill()
+    for c, (o, e) in zip(children, outs):
+        if c.returncode != 0:
+            raise RuntimeError(e[-2000:])
+    ds = [json.loads(o.strip().splitlines()[-1]) for o, _ in outs]
+    sec = max(d["sec"] for d in ds)
+    return {"value": sum(d["bytes"] for d in ds) / sec / 1e9, "unit": "GB/s", "cores": procs,
+            "kind": "oracle", "sec": sec, "reps": reps,
             "sample": f"{n_groups} of {w.batch * w.h_kv} (sequence, kv-head) groups x "
                       f"{w.h_q // w.h_kv} query heads at context {w.seq}, {reps} timed repetitions "
-                      f"({d['sec']:.1f} s); fp64 numpy on one thread, bf16 inputs converted before timing"}
+                      f"({sec:.1f} s) by {procs} concurrent single-threaded processes; fp64 numpy, "
+                      f"bf16 inputs converted before timing"}
 
 
 def run_reference(args, rank):
@@ -494,8 +526,9 @@ def run_reference(args, rank):
         return
     cal = cpu_oracle_decode(w, 1, 5)
     t_group = cal["sec"] / cal["reps"]
-    n_groups = int(max(1, min(w.batch * w.h_kv, 120.0 / (args.steps + args.warmup) / t_group)))
-    res = cpu_oracle_decode(w, n_groups, args.steps, args.warmup)
+    procs = min(host_cores(), w.batch * w.h_kv)
+    n_groups = int(max(1, min(w.batch * w.h_kv, procs * 120.0 / (args.steps + args.warmup) / t_group)))
+    res = cpu_oracle_decode(w, n_groups, args.steps, args.warmup, procs)
     line = {"impl": "reference", "metric": METRIC, "value": res["value"], "unit": "GB/s",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": res["sec"] / args.steps * 1e3,
@@ -679,8 +712,10 @@ def main():
         line["workloads"] = extra
         try:
             cal = cpu_oracle_decode(w, 1, 5)
-            reps = max(1, int(10.0 / (cal["sec"] / cal["reps"] * 16)))
-            line["cpu_baseline"] = cpu_oracle_decode(w, 16, reps) if n == 1 else None
+            procs = min(host_cores(), w.batch * w.h_kv)
+            groups = min(w.batch * w.h_kv, 16 * procs)
+            reps = max(1, int(10.0 / (cal["sec"] / cal["reps"] * groups / procs)))
+            line["cpu_baseline"] = cpu_oracle_decode(w, groups, reps, procs=procs) if n == 1 else None
         except Exception as e:  # reported, not fatal
             line["cpu_baseline"] = {"error": str(e)[-300:]}
     if rank == 0:
