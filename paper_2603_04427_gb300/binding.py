@@ -209,15 +209,14 @@ def decode_workspace(desc: tk_cache_desc, max_seq_len: int, device="cuda") -> to
 
 def tk_attn_decode(cache: ThinKeyCache, q, seq_lens, max_seq_len: int, out, workspace,
                    scale: float | None = None, stream=None):
-    """One decode step: q [B, H_q, r] bf16 -> out [B, H_q, d_v] (fp32 or bf16)."""
+    """One decode step: q [B, H_q, r] bf16 -> out [B, H_q, d_v] (fp32 or bf16, on the GPU or
+    in page-locked host memory, which the kernel then writes directly)."""
     d = cache.desc
     dev = cache.k.device
     _need(q, torch.bfloat16, "q", dev)
     _need(seq_lens, torch.int32, "seq_lens", dev)
     _need(workspace, torch.uint8, "workspace", dev)
-    if out.dtype not in (torch.float32, torch.bfloat16):
-        raise TypeError("out must be float32 or bfloat16")
-    _need(out, out.dtype, "out", dev)
+    _need_out(out, "out", dev)
     if tuple(q.shape) != (d.batch, d.h_q, d.r) or tuple(out.shape) != (d.batch, d.h_q, d.d_v):
         raise ValueError(f"q {tuple(q.shape)} / out {tuple(out.shape)} do not match the cache")
     scale = 1.0 / math.sqrt(d.r) if scale is None else float(scale)
@@ -443,9 +442,7 @@ def tk_attn_decode_noalloc(cache: ThinKeyCache, q, seq_lens, max_seq_len: int, o
     dev = cache.k.device
     _need(q, torch.bfloat16, "q", dev)
     _need(seq_lens, torch.int32, "seq_lens", dev)
-    if out.dtype not in (torch.float32, torch.bfloat16):
-        raise TypeError("out must be float32 or bfloat16")
-    _need(out, out.dtype, "out", dev)
+    _need_out(out, "out", dev)
     if tuple(q.shape) != (d.batch, d.h_q, d.r) or tuple(out.shape) != (d.batch, d.h_q, d.d_v):
         raise ValueError(f"q {tuple(q.shape)} / out {tuple(out.shape)} do not match the cache")
     scale = 1.0 / math.sqrt(d.r) if scale is None else float(scale)

@@ -85,6 +85,26 @@ def test_decode_bf16_output_and_determinism():
     parity(f64(o1), _oracle(cache, q, kn, lens, 1 / math.sqrt(r)), what="bf16 out")
 
 
+@pytest.mark.parametrize("out_dtype", [torch.float32, torch.bfloat16])
+def test_zero_copy_host_output_equals_device_output(out_dtype):
+    """`out` in page-locked host memory: the kernel writes it directly, same bits."""
+    require_gpu()
+    B, hq, hkv, r, dv = 3, 16, 4, 32, 128
+    lens = [2000, 1531, 64]
+    cache, _, _ = _contiguous(B, hq, hkv, r, dv, 2048, lens, False, seed=15)
+    q = inputs.normal_bf16((B, hq, r), seed=18, device="cuda")
+    dev = _run(cache, q, lens, out_dtype=out_dtype)
+    sl = torch.tensor(lens, dtype=torch.int32, device="cuda")
+    host = torch.full((B, hq, dv), float("nan"), dtype=out_dtype).pin_memory()
+    tb.tk_attn_decode(cache, q, sl, max(lens), host, tb.decode_workspace(cache.desc, max(lens)))
+    torch.cuda.synchronize()
+    assert tb.tk_get_device_error() == 0
+    assert torch.equal(host, dev.cpu())
+    with pytest.raises(ValueError):   # pageable host memory is refused
+        tb.tk_attn_decode(cache, q, sl, max(lens), torch.empty(B, hq, dv, dtype=out_dtype),
+                          tb.decode_workspace(cache.desc, max(lens)))
+
+
 def _paged_copy(cache, lens, ps, seed):
     """A paged cache holding the same tokens as the contiguous `cache`."""
     d = cache.desc
