@@ -208,6 +208,20 @@ struct Walker {
   }
 };
 
+// CTAs that share T units: about four units each, so that short contexts are
+// not split across CTAs (every split adds a merge); but one unit each when
+// four-unit shares would leave three quarters of the grid idle, so that small
+// batches spread over the GPU.  Measured: a GPT-2-sized step (60 units) 277 ->
+// 215 us per layer of 32 steps with one unit per CTA; one unit per CTA slowed
+// B = 16 at context 256 (512 units) from 7.8 to 11.8 us; shares in between
+// (3.4 units) were slower than both at B = 4, context 512 (11.1 us against
+// 9.1 and 8.8 us), cutting most pairs at two places.
+__device__ __forceinline__ int split_ctas(long long T, int grid) {
+  const long long four = (T + 3) / 4;
+  const long long want = four < grid / 4 ? T : four;
+  return static_cast<int>(min(static_cast<long long>(grid), max(want, 1LL)));
+}
+
 // CTA owning unit u when CTA c owns [floor(c T / N), floor((c+1) T / N)).
 __device__ __forceinline__ int cta_of(long long u, long long T, int N) {
   return static_cast<int>(((u + 1) * N - 1) / T);
@@ -392,7 +406,7 @@ __device__ void prefetch_first_chunks(const DecodeParams& p, int lane, int limit
   }
   const long long T = __shfl_sync(0xffffffffu, inc, 31);
   const long long pre = inc - x;
-  const int N = static_cast<int>(min(static_cast<long long>(gridDim.x), max((T + 3) / 4, 1LL)));
+  const int N = split_ctas(T, gridDim.x);
   const int c = blockIdx.x;
   if (T == 0 || c >= N) return;  // warp-uniform
   const long long u_begin = T * c / N, u_end = T * (c + 1) / N;
@@ -500,11 +514,10 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
   }
   __syncthreads();
   const long long T = pre[B];
-  // Partition over N = min(grid, ceil(T / 4)) CTAs: every owning CTA gets at
-  // least one unit (four when the cache is small, so short contexts are not
-  // spread over many CTAs) and the CTAs sharing a pair are consecutive; the
-  // rest own nothing.
-  const int N = static_cast<int>(min(static_cast<long long>(gridDim.x), max((T + 3) / 4, 1LL)));
+  // Partition over N = split_ctas(T, grid) CTAs: every owning CTA gets at
+  // least one unit and the CTAs sharing a pair are consecutive; the rest own
+  // nothing.
+  const int N = split_ctas(T, gridDim.x);
   const long long u_begin = c < N ? T * c / N : T, u_end = c < N ? T * (c + 1) / N : T;
 
   if (warp == kCW) {
