@@ -15,7 +15,7 @@ weights are scalars, so nothing else changes when r != d_v (Section 2.1,
 remark after Eq. 4).  ``scale`` is an explicit argument; the configs use
 1/sqrt(r), the factor Eq. 4 prints.
 
-Readings of points the paper leaves open (each listed in the design doc):
+Readings of points the paper leaves open:
   * GQA head mapping (the paper composes thin keys with GQA, Section 3.4,
     Mistral-7B 32 query / 8 kv heads in Section 3.5): query head h reads
     kv head h // G with G = H_q / H_kv (contiguous groups).
