@@ -122,3 +122,39 @@ def test_decode_bytes_configs():
     assert b == 64 * 8 * 32768 * (32 + 4 + 256)
     # Prefill, B=2, H=32, S=8192, r=32, d_v=128: 6.873e11 FLOPs.
     assert abs(cm.prefill_flops(2, 32, 8192, 32, 128) - 6.873e11) / 6.873e11 < 1e-3
+
+
+def test_llama125m_parameter_counts():
+    # Thinning W_Q and W_K to d_select columns removes 2 d_model (d_model - d_select)
+    # weights per layer; W_V and everything else is unchanged (Experiment 6).
+    t = GOLD["llama125m_params"]
+    d, H, L = t["d_model"], t["n_heads"], t["n_layers"]
+    base = t["rows"][0]["params_M"]
+    for row in t["rows"]:
+        r = row["d_select"] // H
+        assert r == row["per_head"]
+        saved = cm.projection_bytes_saved(d, H, H, d // H, r, L, beta=1)
+        assert saved == 2 * L * d * (d - row["d_select"])
+        # both the baseline and the row are printed to 0.1 M
+        assert abs(base - saved / 1e6 - row["params_M"]) <= 0.1, (row, saved)
+        # "QK saved" = 1 - d_select / d_model; 87.5 % is printed as 87, so allow half a unit
+        assert abs(100 * (1 - row["d_select"] / d) - row["qk_saved_pct"]) <= 0.5
+
+
+def test_kv_methods_budget_per_token_and_layer():
+    t = GOLD["kv_methods_budget"]
+    d, H, dh, L = t["d_model"], t["n_heads"], t["d_head"], t["n_layers"]
+    full = cm.c_kv(1, H, dh, 1, beta=1)
+    assert full == t["mha"]["kv_budget"]
+    assert cm.kv_cache_bytes(1, d, 1, 1)["total"] == full
+    for row in t["thin"]:
+        r = row["d_select"] // H
+        got = cm.c_kv_thin(1, H, r, dh, 1, beta=1)
+        assert got == row["kv_budget"] == cm.kv_cache_bytes(1, d, 1, 1, d_select=row["d_select"])["total"]
+        assert abs(100 * (1 - got / full) - row["saved_pct"]) <= 0.05
+        saved = cm.projection_bytes_saved(d, H, H, dh, r, L, beta=1)
+        assert abs(t["mha"]["params_M"] - saved / 1e6 - row["params_M"]) <= 0.1
+    for row in t["gqa"]:
+        got = cm.c_kv(1, row["n_kv_heads"], dh, 1, beta=1)
+        assert got == row["kv_budget"]
+        assert abs(100 * (1 - got / full) - row["saved_pct"]) <= 0.05
