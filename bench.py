@@ -625,7 +625,7 @@ def main():
     e2e_dt, h2d, d2h = measure_decode_e2e(rig, min(args.steps, 5000))
     (e2e_dt,) = max_over_ranks(dist, (e2e_dt,), device)
     achieved = (rig.kv_bytes + rig.io_bytes) / sec_dec / 1e9
-    dec_hash = source_hash("decode.cu", "common.cuh")
+    dec_hash = source_hash("decode.cu", "common.cuh", "kv_row.cuh", "kernels.h")
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": n, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": sec_step * 1e3, "higher_is_better": True,
