@@ -233,8 +233,14 @@ class DecodeRig:
         self.tb.tk_attn_decode(c["cache"], c["q"], c["seq_dec"], self.max_len, c["out"], c["ws"])
 
 
-def graph_time(torch, enqueue, steps, warmup, max_graph=256):
-    """Time exactly `steps` calls of enqueue(i) replayed from CUDA graphs; returns seconds."""
+def graph_time(torch, enqueue, steps, warmup, max_graph=256, min_seconds=0.0, info=None):
+    """Seconds for exactly `steps` calls of enqueue(i), replayed from CUDA graphs.
+
+    One block = the `steps` calls between two CUDA events on the launching
+    stream.  With min_seconds > 0 blocks are replayed back to back until that
+    much device time has passed, and the median block is returned (so that a
+    short block is not decided by one replay, and clock samplers see load);
+    `info` then receives the block count and the device time spanned."""
     stream = torch.cuda.Stream()
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
@@ -256,27 +262,43 @@ def graph_time(torch, enqueue, steps, warmup, max_graph=256):
     full, rem = divmod(steps, G)
     g_full = graph_of(G) if full else None
     g_rem = graph_of(rem) if rem else None
-    with torch.cuda.stream(stream):   # one untimed replay uploads the graphs
+
+    def block():
         if g_full is not None:
-            g_full.replay()
+            for _ in range(full):
+                g_full.replay()
         if g_rem is not None:
             g_rem.replay()
+
+    with torch.cuda.stream(stream):   # one untimed replay uploads the graphs
+        block()
     torch.cuda.synchronize()
-    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with torch.cuda.stream(stream):
-        t0.record(stream)
-        for _ in range(full):
-            g_full.replay()
-        if g_rem is not None:
-            g_rem.replay()
-        t1.record(stream)
-    t1.synchronize()
-    return t0.elapsed_time(t1) / 1e3
+    times = []
+    spent = 0.0
+    while True:
+        # a batch of blocks, each between its own pair of events
+        n_blk = 1 if not times else max(1, min(512, int(len(times) * (min_seconds - spent) / spent) + 1))
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(n_blk + 1)]
+        with torch.cuda.stream(stream):
+            evs[0].record(stream)
+            for j in range(n_blk):
+                block()
+                evs[j + 1].record(stream)
+        evs[-1].synchronize()
+        new = [evs[j].elapsed_time(evs[j + 1]) / 1e3 for j in range(n_blk)]
+        times += new
+        spent += sum(new)
+        if spent >= min_seconds:
+            break
+    if info is not None:
+        info.update(blocks=len(times), timed_region_s=spent)
+    return statistics.median(times)
 
 
-def measure_decode(rig, steps, warmup, mode="fused"):
+def measure_decode(rig, steps, warmup, mode="fused", min_seconds=0.0, info=None):
     torch = rig.torch
-    sec = graph_time(torch, lambda i: rig.step(i, mode), steps, warmup)
+    sec = graph_time(torch, lambda i: rig.step(i, mode), steps, warmup, min_seconds=min_seconds,
+                     info=info)
     return sec / steps
 
 
@@ -342,7 +364,7 @@ def measure_prefill(w, iters, device, torch):
         q, k, v, o = sets[i % len(sets)]
         tb.tk_attn_prefill(q, k, v, o)
 
-    sec = graph_time(torch, enq, iters, 3, max_graph=16) / iters
+    sec = graph_time(torch, enq, iters, 3, max_graph=16, min_seconds=0.5) / iters
     flops = cm.prefill_flops(B, hq, S, r, dv, causal=True)
     return {"ms": sec * 1e3, "tflops": flops / sec / 1e12, "flops_per_launch": flops}
 
@@ -367,7 +389,7 @@ def measure_chunked_prefill(w, iters, device, torch):
     def enq(_):  # the same chunk re-appended at the same positions every time
         tb.tk_attn_prefill_cached(cache, q, kn, vn, sl, L0 + S, out)
 
-    sec = graph_time(torch, enq, iters, 3, max_graph=16) / iters
+    sec = graph_time(torch, enq, iters, 3, max_graph=16, min_seconds=0.3) / iters
     flops = cm.prefill_flops(B, hq, S, r, dv, cached=L0)
     return {"ms": sec * 1e3, "tflops": flops / sec / 1e12, "flops_per_call": flops,
             "cached": L0, "launches": 2}
@@ -396,7 +418,7 @@ def measure_backward(w, iters, device, torch):
     def enq(_):
         tb.tk_attn_backward(q, k, v, out, do, lse, dq, dk, dvv, ws)
 
-    sec = graph_time(torch, enq, iters, 3, max_graph=8) / iters
+    sec = graph_time(torch, enq, iters, 3, max_graph=8, min_seconds=0.3) / iters
     pairs = cm.causal_pairs(S) * B * hq
     flops = pairs * 2 * (3 * r + 2 * dv)   # S^T, dP^T, dV, dK, dQ products
     return {"ms": sec * 1e3, "tflops": flops / sec / 1e12, "flops_per_call": flops, "launches": 2}
@@ -445,24 +467,65 @@ import json, sys, time, os
 sys.path.insert(0, os.environ["TK_ROOT"])
 import torch
 from oracle import attention as oa
+from oracle import cache as oc
 from oracle.attention import bf16_bits_to_f64
 from paper_2603_04427_gb300 import inputs, cost_model as cm
-B, hq, hkv, r, dv, L, seed, n_groups, reps, warm = [int(x) for x in sys.argv[1:11]]
-G = hq // hkv
-# a bounded sample: n_groups (sequence, kv head) groups of the workload, G query heads each
+spec = json.loads(sys.argv[1])
 f = lambda t: bf16_bits_to_f64(t.view(torch.int16).numpy())
-k = f(inputs.normal_bf16((1, n_groups, L, r), seed + 1))
-v = f(inputs.normal_bf16((1, n_groups, L, dv), seed + 2))
-q = f(inputs.normal_bf16((1, n_groups * G, r), seed + 3))
+seed, reps, warm, r, dv = spec["seed"], spec["reps"], spec["warm"], spec["r"], spec["dv"]
+scale = 1.0 / r ** 0.5
+if spec["mode"] == "decode":
+    # a bounded sample: n_groups (sequence, kv head) groups of the workload, G query heads each
+    n, L, G, kf = spec["groups"], spec["L"], spec["G"], spec.get("k", "bf16")
+    kb = inputs.normal_bf16((1, n, L, r), seed + 1)
+    v = f(inputs.normal_bf16((1, n, L, dv), seed + 2))
+    q = f(inputs.normal_bf16((1, n * G, r), seed + 3))
+    if kf == "bf16":
+        k, sc, kbytes, sbytes = f(kb), None, 2, 0
+    else:   # the oracle's own quantiser, before timing
+        quant = oc.quantize_int8_per_token if kf == "int8" else oc.quantize_int4_per_token
+        k, sc = quant(kb.float().numpy())
+        kbytes, sbytes = (1, 4) if kf == "int8" else (0.5, 4)
+    work = lambda: oa.attention_decode(q, k, v, [L], scale, k_scale=sc)
+    amount = cm.decode_kv_bytes([L] * n, 1, r, dv, k_bytes=kbytes, k_scale_bytes=sbytes)
+elif spec["mode"] == "decode_seq":
+    # groups of different context lengths, built and timed one after the other
+    G, kf, el, amount = spec["G"], spec.get("k", "bf16"), 0.0, 0
+    print("ready", flush=True)
+    sys.stdin.readline()
+    for i, L in enumerate(spec["Ls"]):
+        kb = inputs.normal_bf16((1, 1, L, r), seed + 10 * i + 1)
+        v = f(inputs.normal_bf16((1, 1, L, dv), seed + 10 * i + 2))
+        q = f(inputs.normal_bf16((1, G, r), seed + 10 * i + 3))
+        if kf == "bf16":
+            k, sc, kbytes, sbytes = f(kb), None, 2, 0
+        else:
+            quant = oc.quantize_int8_per_token if kf == "int8" else oc.quantize_int4_per_token
+            k, sc = quant(kb.float().numpy())
+            kbytes, sbytes = (1, 4) if kf == "int8" else (0.5, 4)
+        t0 = time.perf_counter()
+        oa.attention_decode(q, k, v, [L], scale, k_scale=sc)
+        el += time.perf_counter() - t0
+        amount += cm.decode_kv_bytes([L], 1, r, dv, k_bytes=kbytes, k_scale_bytes=sbytes)
+    print(json.dumps({"sec": el, "reps": 1, "amount": amount}))
+    sys.exit(0)
+else:
+    # a bounded sample of prefill: query rows row0 .. row0 + n - 1 of one causal head
+    row0, n = spec["row0"], spec["rows"]
+    q = f(inputs.normal_bf16((n, r), seed + 1))
+    k = f(inputs.normal_bf16((row0 + n, r), seed + 2))
+    v = f(inputs.normal_bf16((row0 + n, dv), seed + 3))
+    work = lambda: oa.attention_head(q, k, v, scale, causal_offset=row0)
+    amount = sum(i + 1 for i in range(row0, row0 + n)) * 2 * (r + dv)
 print("ready", flush=True)   # inputs built; the timed work starts on the parent's word
 sys.stdin.readline()
 for _ in range(warm):
-    oa.attention_decode(q, k, v, [L], 1.0 / r ** 0.5)
+    work()
 t0 = time.perf_counter()
 for _ in range(reps):
-    oa.attention_decode(q, k, v, [L], 1.0 / r ** 0.5)
+    work()
 el = time.perf_counter() - t0
-print(json.dumps({"sec": el, "reps": reps, "bytes": cm.decode_kv_bytes([L] * n_groups, 1, r, dv) * reps}))
+print(json.dumps({"sec": el, "reps": reps, "amount": amount * reps}))
 """
 
 
@@ -473,21 +536,14 @@ def host_cores() -> int:
         return os.cpu_count() or 1
 
 
-def cpu_oracle_decode(w, n_groups: int, reps: int, warmup: int = 1, procs: int = 1):
-    """Time `reps` oracle decodes of a sample of the workload: `procs` fresh
-    single-threaded processes, each on its share of the n_groups (sequence, kv
-    head) groups, start their timed loops together; throughput = all their
-    bytes / the slowest one's time."""
-    procs = max(1, min(procs, n_groups))
-    shares = [n_groups // procs + (1 if k < n_groups % procs else 0) for k in range(procs)]
+def _run_cpu_children(specs):
+    """Fresh single-threaded oracle processes, one per spec, built first and then
+    started together; returns their results (seconds, repetitions, amount of work)."""
     env = dict(os.environ, TK_ROOT=ROOT, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1",
                MKL_NUM_THREADS="1", CUDA_VISIBLE_DEVICES="")
-    children = []
-    for k, share in enumerate(shares):
-        args = [str(x) for x in (w.batch, w.h_q, w.h_kv, w.r, w.d_v, w.seq, w.seed + 7 * k, share, reps, warmup)]
-        children.append(subprocess.Popen([sys.executable, "-c", CPU_CHILD] + args, env=env, text=True,
-                                         stdin=subprocess.PIPE, stdout=subprocess.PIPE,
-                                         stderr=subprocess.PIPE))
+    children = [subprocess.Popen([sys.executable, "-c", CPU_CHILD, json.dumps(sp)], env=env,
+                                 text=True, stdin=subprocess.PIPE, stdout=subprocess.PIPE,
+                                 stderr=subprocess.PIPE) for sp in specs]
     try:
         for c in children:   # every child has built its inputs
             if c.stdout.readline().strip() != "ready":
@@ -503,14 +559,103 @@ def cpu_oracle_decode(w, n_groups: int, reps: int, warmup: int = 1, procs: int =
     for c, (o, e) in zip(children, outs):
         if c.returncode != 0:
             raise RuntimeError(e[-2000:])
-    ds = [json.loads(o.strip().splitlines()[-1]) for o, _ in outs]
+    return [json.loads(o.strip().splitlines()[-1]) for o, _ in outs]
+
+
+def cpu_oracle_decode(w, n_groups: int, reps: int, warmup: int = 1, procs: int = 1, L=None,
+                      k_fmt=None, r=None):
+    """Time `reps` oracle decodes of a sample of the workload: `procs` fresh
+    single-threaded processes, each on its share of the n_groups (sequence, kv
+    head) groups, start their timed loops together; throughput = all their
+    bytes / the slowest one's time."""
+    procs = max(1, min(procs, n_groups))
+    shares = [n_groups // procs + (1 if k < n_groups % procs else 0) for k in range(procs)]
+    L = L or w.seq
+    r = r or w.r
+    k_fmt = k_fmt or ("int8" if w.k_int8 else "bf16")
+    ds = _run_cpu_children([dict(mode="decode", seed=w.seed + 7 * k, reps=reps, warm=warmup, r=r,
+                                 dv=w.d_v, groups=share, L=L, G=w.h_q // w.h_kv, k=k_fmt)
+                            for k, share in enumerate(shares)])
     sec = max(d["sec"] for d in ds)
-    return {"value": sum(d["bytes"] for d in ds) / sec / 1e9, "unit": "GB/s", "cores": procs,
+    return {"value": sum(d["amount"] for d in ds) / sec / 1e9, "unit": "GB/s", "cores": procs,
             "kind": "oracle", "sec": sec, "reps": reps,
             "sample": f"{n_groups} of {w.batch * w.h_kv} (sequence, kv-head) groups x "
-                      f"{w.h_q // w.h_kv} query heads at context {w.seq}, {reps} timed repetitions "
-                      f"({sec:.1f} s) by {procs} concurrent single-threaded processes; fp64 numpy, "
-                      f"bf16 inputs converted before timing"}
+                      f"{w.h_q // w.h_kv} query heads at context {L} ({k_fmt} keys, r={r}), "
+                      f"{reps} timed repetitions ({sec:.1f} s) by {procs} concurrent "
+                      f"single-threaded processes; fp64 numpy, inputs converted before timing"}
+
+
+def cpu_oracle_prefill(w, rows: int, reps: int, procs: int, warmup: int = 1):
+    """Time the oracle's causal prefill on a sample of the workload: process p computes
+    `rows` consecutive query rows of one head, its blocks spread evenly over the
+    sequence (so the sample holds short and long rows); throughput = the unmasked
+    pairs' FLOPs (2 (r + d_v) per pair) of all processes / the slowest one's time."""
+    S = w.seq
+    starts = [((S - rows) * p // max(1, procs - 1)) // 16 * 16 for p in range(procs)]
+    ds = _run_cpu_children([dict(mode="prefill", seed=w.seed + 7 * p, reps=reps, warm=warmup,
+                                 r=w.r, dv=w.d_v, row0=r0, rows=rows)
+                            for p, r0 in enumerate(starts)])
+    sec = max(d["sec"] for d in ds)
+    flops = sum(d["amount"] for d in ds)
+    total = w.batch * w.h_q * S * (S + 1) // 2 * 2 * (w.r + w.d_v)
+    return {"value": flops / sec / 1e12, "unit": "TFLOP/s", "cores": procs, "kind": "oracle",
+            "sec": sec, "reps": reps,
+            "full_workload_s_extrapolated": total / (flops / sec) if flops else None,
+            "sample": f"{procs} blocks of {rows} consecutive causal query rows (one head each, "
+                      f"starting rows spread over 0..{S - rows}) of the {w.batch}x{w.h_q}-head "
+                      f"S={S} prefill, {reps} timed repetitions ({sec:.1f} s) by {procs} "
+                      f"concurrent single-threaded processes; fp64 numpy"}
+
+
+def cpu_oracle_workloads():
+    """The oracle's time on every workload (fp64 numpy, all host cores): measured in
+    full where that takes seconds, else on a stated sample and extrapolated by the
+    workload's work.  Reported in one JSON line by ``bench.py --only cpu``."""
+    from paper_2603_04427_gb300 import inputs
+    from paper_2603_04427_gb300 import workloads as wl
+    cores = host_cores()
+    res = {}
+
+    def spread(items, procs):
+        return [items[p::procs] for p in range(procs) if items[p::procs]]
+
+    # GPT-2-small layer: 12 heads' causal prefill of 256 rows, then 32 decode steps
+    g = wl.GPT2_LAYER
+    pre = _run_cpu_children([dict(mode="prefill", seed=g.seed + p, reps=1, warm=1, r=g.r, dv=g.d_v,
+                                  row0=0, rows=g.seq) for p in range(g.h_q)])
+    steps = [g.seq + t + 1 for t in range(g.decode_steps)]
+    dec = _run_cpu_children([dict(mode="decode_seq", seed=g.seed + 50 + p, reps=1, warm=0, r=g.r,
+                                  dv=g.d_v, G=1, Ls=steps) for p in range(g.h_q)])
+    res[g.name] = {"sec": max(d["sec"] for d in pre) + max(d["sec"] for d in dec),
+                   "cores": g.h_q, "how": "measured in full (one process per head)"}
+    # Mistral GQA decode: all 128 (sequence, kv head) groups
+    m = wl.MISTRAL_GQA_DECODE
+    d = cpu_oracle_decode(m, m.batch * m.h_kv, 1, 1, min(cores, m.batch * m.h_kv))
+    res[m.name] = {"sec": d["sec"], "cores": d["cores"], "how": "measured in full"}
+    # 7B prefill: blocks of 512 query rows spread over the sequence, extrapolated by FLOPs
+    p7 = cpu_oracle_prefill(wl.MHA7B_PREFILL, 512, 1, cores)
+    res[wl.MHA7B_PREFILL.name] = {"sec": p7["full_workload_s_extrapolated"], "cores": cores,
+                                  "how": "extrapolated from " + p7["sample"]}
+    # paged long-context decode: all 32 (sequence, kv head) groups at their drawn lengths
+    pw = wl.PAGED_LONG_DECODE
+    lens = inputs.uniform_lengths(pw.batch, pw.seq_range[0], pw.seq_range[1], seed=pw.seed)
+    items = [lens[b] for b in range(pw.batch) for _ in range(pw.h_kv)]
+    dd = _run_cpu_children([dict(mode="decode_seq", seed=pw.seed + 13 * p, reps=1, warm=0, r=pw.r,
+                                 dv=pw.d_v, G=pw.h_q // pw.h_kv, Ls=part)
+                            for p, part in enumerate(spread(items, min(cores, len(items))))])
+    res[pw.name] = {"sec": max(x["sec"] for x in dd), "cores": len(dd),
+                    "how": "measured in full (gathered contexts; the oracle's gather not timed)"}
+    # int8 keys, B=64, context 32768: two groups per core, extrapolated to all 512 groups
+    iw = wl.INT8_DECODE
+    n_s = 2 * cores
+    dd = _run_cpu_children([dict(mode="decode_seq", seed=iw.seed + 13 * p, reps=1, warm=0, r=iw.r,
+                                 dv=iw.d_v, G=iw.h_q // iw.h_kv, k="int8", Ls=[iw.seq, iw.seq])
+                            for p in range(cores)])
+    sec = max(x["sec"] for x in dd)
+    res[iw.name] = {"sec": sec * iw.batch * iw.h_kv / n_s, "cores": cores,
+                    "how": f"extrapolated from {n_s} of {iw.batch * iw.h_kv} (sequence, kv head) "
+                           f"groups ({sec:.2f} s, two per core)"}
+    return res
 
 
 def run_reference(args, rank):
@@ -561,8 +706,10 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--headline-only", action="store_true",
                     help="skip the secondary workloads and the CPU baseline")
-    ap.add_argument("--only", choices=("prefill", "chunked", "backward", "gpt2", "paged", "int8"),
-                    help="run one secondary workload alone (for profiling) and print its result")
+    ap.add_argument("--only", choices=("prefill", "chunked", "backward", "gpt2", "paged", "int8",
+                                       "cpu"),
+                    help="run one secondary workload alone (for profiling) and print its result; "
+                         "cpu: the oracle's time on every workload")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -572,6 +719,9 @@ def main():
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         run_reference(args, rank)
+        return
+    if args.only == "cpu":
+        print(json.dumps({"only": "cpu", "oracle_seconds": cpu_oracle_workloads()}), flush=True)
         return
 
     import torch
@@ -614,9 +764,12 @@ def main():
     torch.cuda.synchronize()
     clocks = ClockSampler(local)
     clocks.start()
-    sec_step = measure_decode(rig, args.steps, args.warmup, mode="fused")
-    sec_two = measure_decode(rig, args.steps, args.warmup, mode="append")
-    sec_dec = measure_decode(rig, args.steps, args.warmup, mode="decode")
+    timing = {}
+    # the headline: K-step blocks replayed for at least a second, median block
+    sec_step = measure_decode(rig, args.steps, args.warmup, mode="fused", min_seconds=1.0,
+                              info=timing)
+    sec_two = measure_decode(rig, args.steps, args.warmup, mode="append", min_seconds=0.2)
+    sec_dec = measure_decode(rig, args.steps, args.warmup, mode="decode", min_seconds=0.3)
     torch.cuda.synchronize()
     clk = clocks.stop()
     sec_step, sec_dec, sec_two = max_over_ranks(dist, (sec_step, sec_dec, sec_two), device)
@@ -653,32 +806,30 @@ def main():
                        "buffer (tk_copy_async) and the fused append + decode, issued as one "
                        "prepared binding call; the kernel writes the output into page-locked "
                        "host memory (zero-copy); host synchronisation every step"},
-        "gpu_launches": args.steps,
+        "gpu_launches": args.steps * timing.get("blocks", 1),
+        "timing": {"blocks": timing.get("blocks"), "timed_region_s": timing.get("timed_region_s"),
+                   "launches_per_step": 1,
+                   "ms_per_step": f"median over blocks of {args.steps} steps (CUDA events)"},
         "clocks": clk,
     }
     del rig
     torch.cuda.empty_cache()
 
     if rank == 0 and not args.headline_only:
+        def r3(x):
+            return float(f"{x:.4g}")
+        if n == 1:
+            try:
+                cal = cpu_oracle_decode(w, 1, 5)
+                procs = min(host_cores(), w.batch * w.h_kv)
+                groups = min(w.batch * w.h_kv, 16 * procs)
+                reps = max(1, int(10.0 / (cal["sec"] / cal["reps"] * groups / procs)))
+                line["cpu_baseline"] = cpu_oracle_decode(w, groups, reps, procs=procs)
+            except Exception as e:  # reported, not fatal
+                line["cpu_baseline"] = {"error": str(e)[-300:]}
+        else:
+            line["cpu_baseline"] = None
         extra = {}
-        # causal prefill, B=2, H=32, S=8192, r=32, d_v=128, bf16 out
-        pw = wl.MHA7B_PREFILL
-        pf = measure_prefill(pw, 20, device, torch)
-        if "tflops" in pf:
-            pf.update(frac=pf["tflops"] / peaks["bf16_tflops"], peak=peaks["bf16_tflops"],
-                      peak_source=peak_src, bound="tensor",
-                      traffic=recorded_traffic("prefill", pw.name,
-                                               source_hash("prefill.cu", "common.cuh", "tc05.cuh")))
-        extra[pw.name] = dict(pw.as_config(), **pf)
-        bw = measure_backward(pw, 10, device, torch)
-        bw.update(frac=bw["tflops"] / peaks["bf16_tflops"], peak=peaks["bf16_tflops"],
-                  peak_source=peak_src, bound="tensor", kernel="bwd_tc_kernel<32,128> (tcgen05)")
-        extra[pw.name.replace("prefill", "backward")] = dict(pw.as_config(), **bw)
-        cw = wl.CHUNKED_PREFILL
-        cp = measure_chunked_prefill(cw, 20, device, torch)
-        cp.update(frac=cp["tflops"] / peaks["bf16_tflops"], peak=peaks["bf16_tflops"],
-                  peak_source=peak_src, bound="tensor")
-        extra[cw.name] = dict(cw.as_config(), **cp)
         gw = wl.GPT2_LAYER
         extra[gw.name] = dict(gw.as_config(), **measure_gpt2_layer(gw, 50, device, torch))
         # paged long-context decode
@@ -687,14 +838,14 @@ def main():
         s = measure_decode(prig, 200, 20, mode="fused")
         sd = measure_decode(prig, 200, 20, mode="decode")
         extra[pl.name] = dict(pl.as_config(), seq_lens=prig.lens, kv_bytes=prig.kv_bytes,
-                              step_us=s * 1e6, gbs=prig.kv_bytes / s / 1e9,
-                              decode_kernel_us=sd * 1e6,
-                              decode_kernel_frac=(prig.kv_bytes + prig.io_bytes) / sd / 1e9 / peaks["hbm_gbs"])
+                              step_us=r3(s * 1e6), gbs=r3(prig.kv_bytes / s / 1e9),
+                              decode_kernel_us=r3(sd * 1e6),
+                              decode_kernel_frac=r3((prig.kv_bytes + prig.io_bytes) / sd / 1e9 / peaks["hbm_gbs"]))
         del prig
         torch.cuda.empty_cache()
-        # int8 keys, B=64, context 32768, and the r sweep (int8 and bf16 keys)
+        # quantised keys, B=64, context 32768, and the r sweep (int4, int8 and bf16 keys)
         iw = wl.INT8_DECODE
-        sweep = []
+        rows = []
         for r in iw.r_sweep:
             for kf in ("int4", "int8", "bf16"):
                 if kf == "int4" and r < 32:
@@ -702,22 +853,49 @@ def main():
                 rr = DecodeRig(iw, device, copies=1, k_fmt=kf, r=r)
                 s = measure_decode(rr, 50, 5, mode="fused")
                 sd = measure_decode(rr, 50, 5, mode="decode")
-                sweep.append({"r": r, "k_dtype": kf, "kv_bytes": rr.kv_bytes,
-                              "step_us": s * 1e6, "gbs": rr.kv_bytes / s / 1e9,
-                              "decode_kernel_us": sd * 1e6,
-                              "decode_kernel_frac": (rr.kv_bytes + rr.io_bytes) / sd / 1e9 / peaks["hbm_gbs"]})
+                rows.append([r, kf, rr.kv_bytes, r3(s * 1e6), r3(rr.kv_bytes / s / 1e9), r3(sd * 1e6),
+                             r3((rr.kv_bytes + rr.io_bytes) / sd / 1e9 / peaks["hbm_gbs"])])
                 del rr
                 torch.cuda.empty_cache()
-        extra[iw.name] = dict(iw.as_config(), sweep=sweep)
+        extra[iw.name] = dict(iw.as_config(), sweep={
+            "cols": ["r", "k_dtype", "kv_bytes", "step_us", "GB/s", "decode_kernel_us",
+                     "decode_kernel_frac"], "rows": rows})
+        # training backward and chunked prefill of the 7B shape
+        pw = wl.MHA7B_PREFILL
+        bw = measure_backward(pw, 10, device, torch)
+        extra[pw.name.replace("prefill", "backward")] = dict(
+            pw.as_config(), kernel="bwd_tc_kernel<32,128> (tcgen05)", ms=r3(bw["ms"]),
+            tflops=r3(bw["tflops"]), frac=r3(bw["tflops"] / peaks["bf16_tflops"]),
+            flops_per_call=bw["flops_per_call"], launches=bw["launches"])
+        cw = wl.CHUNKED_PREFILL
+        cp = measure_chunked_prefill(cw, 20, device, torch)
+        extra[cw.name] = dict(cw.as_config(), ms=r3(cp["ms"]), tflops=r3(cp["tflops"]),
+                              frac=r3(cp["tflops"] / peaks["bf16_tflops"]),
+                              flops_per_call=cp["flops_per_call"], launches=cp["launches"])
         line["workloads"] = extra
-        try:
-            cal = cpu_oracle_decode(w, 1, 5)
-            procs = min(host_cores(), w.batch * w.h_kv)
-            groups = min(w.batch * w.h_kv, 16 * procs)
-            reps = max(1, int(10.0 / (cal["sec"] / cal["reps"] * groups / procs)))
-            line["cpu_baseline"] = cpu_oracle_decode(w, groups, reps, procs=procs) if n == 1 else None
-        except Exception as e:  # reported, not fatal
-            line["cpu_baseline"] = {"error": str(e)[-300:]}
+        # the causal prefill half of the metric, last on the line
+        pf = measure_prefill(pw, 20, device, torch)
+        pre = dict(pw.as_config(), kernel="prefill_kernel<32,128> (tcgen05)")
+        if "tflops" in pf:
+            pre.update(ms=r3(pf["ms"]), tflops=r3(pf["tflops"]), flops_per_launch=pf["flops_per_launch"],
+                       roofline={"bound": "tensor", "achieved": r3(pf["tflops"]),
+                                 "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                                 "frac": r3(pf["tflops"] / peaks["bf16_tflops"]),
+                                 "peak_source": peak_src,
+                                 "traffic": recorded_traffic("prefill", pw.name, source_hash(
+                                     "prefill.cu", "common.cuh", "tc05.cuh"))})
+        else:
+            pre.update(pf)
+        if n == 1:
+            try:
+                procs = host_cores()
+                cal = cpu_oracle_prefill(pw, 512, 1, 1)
+                reps = max(1, int(10.0 / cal["sec"]))
+                cb = cpu_oracle_prefill(pw, 512, reps, procs)
+                pre["cpu_baseline"] = {k: (r3(v) if isinstance(v, float) else v) for k, v in cb.items()}
+            except Exception as e:  # reported, not fatal
+                pre["cpu_baseline"] = {"error": str(e)[-300:]}
+        line["prefill"] = pre
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist:

@@ -298,10 +298,13 @@ tk_status tk_copy_async(void* dst, const void* src, size_t bytes, void* stream);
  *   GPU that loads the library keeps until the process exits.  A shape whose
  *   tk_decode_workspace_size exceeds it is rejected with TK_ERR_WORKSPACE
  *   (tk_last_error gives both sizes) before anything is launched.
- *   No device memory is allocated or freed.  The first call on each device
- *   looks up the array's device address (with that device current) and
- *   caches it; make that first call before any stream capture.  Each call
- *   clears the counters with one cudaMemsetAsync on `stream`.
+ *   No device memory is allocated or freed.  Every call looks up the
+ *   array's device address for the calling thread's current device
+ *   (cudaGetSymbolAddress, which allocates nothing; the first lookup on a
+ *   device may load the library's device code there, so make the first call
+ *   on each device before any stream capture).  A call that passes every
+ *   check clears the counters with one cudaMemsetAsync on `stream` just
+ *   before its launch; a rejected call writes nothing.
  *   All calls on a device share the array and it keeps the last call's
  *   contents: calls that may overlap on the GPU (different streams without
  *   ordering between them) race and give wrong results.                   */
@@ -316,6 +319,17 @@ tk_status tk_attn_decode_noalloc(const tk_cache_desc* desc, const void* q, const
  * last call, else a nonzero code (1 = index out of range, 2 = a wait timed
  * out).  Returns TK_ERR_DEVICE when the word was nonzero.                  */
 tk_status tk_get_device_error(int32_t* code_out, void* stream);
+
+/* Diagnostic of the failure detection (not part of the paper's method).
+ * Every wait inside the library's kernels gives up after 1 s, records code 2
+ * in the device error word and lets its kernel return instead of spinning.
+ * This call exercises that path: it launches one thread that waits, through
+ * the same bounded wait, on an mbarrier that nothing ever arrives at, with a
+ * limit of limit_us microseconds (1 .. 1000000) in place of the 1 s.  The
+ * wait runs out, code 2 is recorded and the kernel returns; the context stays
+ * usable.  The next tk_get_device_error returns TK_ERR_DEVICE with
+ * *code_out == 2.  A limit outside the range gives TK_ERR_INVALID_ARG.     */
+tk_status tk_check_wait_timeout(int32_t limit_us, void* stream);
 
 /* Static string naming a status code.                                      */
 const char* tk_status_string(tk_status status);

@@ -24,7 +24,8 @@ LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtk.so")
 EXPORTED = ("tk_kv_append", "tk_attn_prefill", "tk_decode_workspace_size", "tk_attn_decode",
             "tk_attn_decode_append", "tk_attn_decode_noalloc", "tk_attn_prefill_cached",
             "tk_attn_forward", "tk_backward_workspace_size", "tk_attn_backward", "tk_copy_async",
-            "tk_get_device_error", "tk_status_string", "tk_last_error", "tk_abi_version")
+            "tk_check_wait_timeout", "tk_get_device_error", "tk_status_string", "tk_last_error",
+            "tk_abi_version")
 
 
 class TkError(RuntimeError):
@@ -69,6 +70,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
                                         sz, vp]),
         "tk_attn_decode_noalloc": (i32, [dp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp]),
         "tk_get_device_error": (i32, [ctypes.POINTER(i32), vp]),
+        "tk_check_wait_timeout": (i32, [i32, vp]),
         "tk_copy_async": (i32, [vp, vp, sz, vp]),
         "tk_status_string": (ctypes.c_char_p, [i32]),
         "tk_last_error": (ctypes.c_char_p, []),
@@ -453,6 +455,13 @@ def tk_attn_decode_noalloc(cache: ThinKeyCache, q, seq_lens, max_seq_len: int, o
                                     TK_F32 if out.dtype == torch.float32 else TK_BF16, scale,
                                     _stream(stream)), "tk_attn_decode_noalloc")
     return out
+
+
+def tk_check_wait_timeout(limit_us: int, stream=None):
+    """Run the failure-detection diagnostic: a bounded wait that must run out
+    after limit_us microseconds and record code 2 (see include/tk.h)."""
+    _check(load_library().tk_check_wait_timeout(int(limit_us), _stream(stream)),
+           "tk_check_wait_timeout")
 
 
 def tk_get_device_error(stream=None) -> int:

@@ -69,18 +69,25 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Wait for the phase with the given parity to complete.  Returns false (and
-// records a timeout) if it has not completed within TK_WAIT_LIMIT_NS.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err) {
+// records a timeout) if it has not completed within limit_ns nanoseconds of
+// %globaltimer.
+__device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, int* err,
+                                              uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   while (true) {
     for (int i = 0; i < 64; ++i)
       if (mbar_try_wait(bar, parity)) return true;
-    if (global_timer_ns() - t0 > TK_WAIT_LIMIT_NS) {
+    if (global_timer_ns() - t0 > limit_ns) {
       record_error(err, TK_DEVERR_TIMEOUT);
       return false;
     }
   }
+}
+
+// The wait every kernel uses: at most TK_WAIT_LIMIT_NS.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err) {
+  return mbar_wait_for(bar, parity, err, TK_WAIT_LIMIT_NS);
 }
 
 // ---------------------------------------------------------------- dependent launch

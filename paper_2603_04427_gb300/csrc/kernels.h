@@ -132,4 +132,8 @@ cudaError_t launch_backward_tc(const BackwardParams& p, cudaStream_t stream, int
 
 cudaError_t launch_prefill(const PrefillParams& p, cudaStream_t stream, int* unsupported);
 
+// One thread waits limit_ns on an mbarrier that nothing arrives at, through the
+// library's bounded wait, which records a timeout in *err and returns.
+cudaError_t launch_wait_timeout(int* err, uint64_t limit_ns, cudaStream_t stream);
+
 }  // namespace tk

@@ -22,11 +22,10 @@ __device__ int g_tk_device_error;
 constexpr int kMaxDevices = 64;
 
 struct DeviceInfo {
-  bool ready = false;
   int num_sms = 0;
   int* err = nullptr;  // device address of g_tk_device_error
 };
-DeviceInfo g_dev[kMaxDevices];
+int g_num_sms[kMaxDevices];  // 0 until read
 std::mutex g_dev_mu;
 
 thread_local std::string t_last_error;
@@ -46,23 +45,29 @@ tk_status cuda_fail(cudaError_t e, const char* what) {
   return fail(TK_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
 }
 
-// Per-device set-up (SM count, device address of the error word), done once
-// per device with that device current.
-tk_status device_info(DeviceInfo** out) {
+// Per-call device facts for the current device: its SM count (read once per
+// device and kept) and the device address of the error word.  The address is
+// looked up on every call (cudaGetSymbolAddress allocates nothing): after a
+// cudaDeviceReset the library's device code is loaded again, possibly at
+// another address, and a cached pointer would be stale.
+tk_status device_info(DeviceInfo* out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
   if (dev < 0 || dev >= kMaxDevices) return fail(TK_ERR_UNSUPPORTED, "device ordinal %d", dev);
-  std::lock_guard<std::mutex> lock(g_dev_mu);
-  DeviceInfo& d = g_dev[dev];
-  if (!d.ready) {
-    e = cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
-    e = cudaGetSymbolAddress(reinterpret_cast<void**>(&d.err), g_tk_device_error);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(error word)");
-    d.ready = true;
+  {
+    std::lock_guard<std::mutex> lock(g_dev_mu);
+    if (g_num_sms[dev] == 0) {
+      e = cudaDeviceGetAttribute(&g_num_sms[dev], cudaDevAttrMultiProcessorCount, dev);
+      if (e != cudaSuccess) {
+        g_num_sms[dev] = 0;
+        return cuda_fail(e, "cudaDeviceGetAttribute");
+      }
+    }
+    out->num_sms = g_num_sms[dev];
   }
-  *out = &d;
+  e = cudaGetSymbolAddress(reinterpret_cast<void**>(&out->err), g_tk_device_error);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(error word)");
   return TK_OK;
 }
 
@@ -134,11 +139,11 @@ tk_status tk_kv_append(const tk_cache_desc* desc, void* k_cache, void* v_cache, 
   if (!seq_lens || !k_new || !v_new) return fail(TK_ERR_INVALID_ARG, "seq_lens / k_new / v_new is NULL");
   if (!aligned16(k_new) || !aligned16(v_new))
     return fail(TK_ERR_INVALID_ARG, "k_new / v_new must be 16-byte aligned");
-  DeviceInfo* dev;
+  DeviceInfo dev;
   if ((s = device_info(&dev)) != TK_OK) return s;
   tk::AppendParams p{};
   p.k = k_cache; p.v = v_cache; p.k_scale = k_scale; p.page_table = page_table;
-  p.seq_lens = seq_lens; p.k_new = k_new; p.v_new = v_new; p.err = dev->err;
+  p.seq_lens = seq_lens; p.k_new = k_new; p.v_new = v_new; p.err = dev.err;
   p.B = desc->batch; p.Hkv = desc->h_kv; p.R = desc->r; p.DV = desc->d_v; p.T = n_new;
   p.k_fmt = key_format(desc->k_dtype);
   p.capacity = desc->capacity;
@@ -202,12 +207,12 @@ tk_status tk_attn_backward(const void* q, const void* k, const void* v, const vo
   const size_t need = tk_backward_workspace_size(batch, h_q, seq);
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0 || workspace_bytes < need)
     return fail(TK_ERR_WORKSPACE, "workspace needs %zu bytes, 256-byte aligned", need);
-  DeviceInfo* dev;
+  DeviceInfo dev;
   tk_status s = device_info(&dev);
   if (s != TK_OK) return s;
   tk::BackwardParams p{};
   p.q = q; p.k = k; p.v = v; p.out = out; p.d_out = d_out; p.lse = lse;
-  p.dq = dq; p.dk = dk; p.dv = dv; p.err = dev->err;
+  p.dq = dq; p.dk = dk; p.dv = dv; p.err = dev.err;
   p.S_pad = tk::backward_rows(seq);
   const size_t half = need / 2;   // each array 256-byte aligned
   p.nl2 = static_cast<float*>(workspace);
@@ -239,15 +244,15 @@ tk_status prefill_impl(const void* q, const void* k, const void* v, void* out, f
   if (!q || !k || !v || !out) return fail(TK_ERR_INVALID_ARG, "q / k / v / out is NULL");
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out))
     return fail(TK_ERR_INVALID_ARG, "q / k / v / out must be 16-byte aligned");
-  DeviceInfo* dev;
+  DeviceInfo dev;
   tk_status s = device_info(&dev);
   if (s != TK_OK) return s;
   tk::PrefillParams p{};
-  p.q = q; p.k = k; p.v = v; p.out = out; p.out_f32 = out_dtype == TK_F32; p.err = dev->err;
+  p.q = q; p.k = k; p.v = v; p.out = out; p.out_f32 = out_dtype == TK_F32; p.err = dev.err;
   p.B = batch; p.Hq = h_q; p.Hkv = h_kv; p.S = seq; p.R = r; p.DV = d_v;
   p.causal = causal != 0;
   p.scale_log2 = scale * 1.4426950408889634f;
-  p.num_sms = dev->num_sms;
+  p.num_sms = dev.num_sms;
   p.lse = lse;
   int uns = 0;
   cudaError_t e = tk::launch_prefill(p, static_cast<cudaStream_t>(stream), &uns);
@@ -279,13 +284,13 @@ tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void*
     return fail(TK_ERR_INVALID_ARG, "q / out / seq_lens / k_new / v_new is NULL");
   if (!aligned16(q) || !aligned16(out) || !aligned16(k_new) || !aligned16(v_new))
     return fail(TK_ERR_INVALID_ARG, "q / out / k_new / v_new must be 16-byte aligned");
-  DeviceInfo* dev;
+  DeviceInfo dev;
   if ((s = device_info(&dev)) != TK_OK) return s;
   const cudaStream_t st = static_cast<cudaStream_t>(stream);
   // 1. the chunk's keys and values into the cache at seq_lens[b]
   tk::AppendParams a{};
   a.k = k_cache; a.v = v_cache; a.k_scale = nullptr; a.page_table = page_table;
-  a.seq_lens = seq_lens; a.k_new = k_new; a.v_new = v_new; a.err = dev->err;
+  a.seq_lens = seq_lens; a.k_new = k_new; a.v_new = v_new; a.err = dev.err;
   a.B = desc->batch; a.Hkv = desc->h_kv; a.R = desc->r; a.DV = desc->d_v; a.T = seq;
   a.k_fmt = 0;
   a.capacity = desc->capacity;
@@ -299,12 +304,12 @@ tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void*
   // 2. the chunk's queries over the cache's first seq_lens[b] + seq tokens
   tk::PrefillParams p{};
   p.q = q; p.k = k_cache; p.v = v_cache; p.out = out; p.out_f32 = out_dtype == TK_F32;
-  p.err = dev->err;
+  p.err = dev.err;
   p.B = desc->batch; p.Hq = desc->h_q; p.Hkv = desc->h_kv; p.S = seq; p.R = desc->r;
   p.DV = desc->d_v;
   p.causal = causal != 0;
   p.scale_log2 = scale * 1.4426950408889634f;
-  p.num_sms = dev->num_sms;
+  p.num_sms = dev.num_sms;
   p.seq_lens = seq_lens;
   p.page_table = page_table;
   p.capacity = desc->capacity;
@@ -325,10 +330,10 @@ tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void*
 
 size_t tk_decode_workspace_size(const tk_cache_desc* desc, int32_t max_seq_len) {
   if (check_desc(desc) != TK_OK || max_seq_len < 0) return 0;
-  DeviceInfo* dev;
+  DeviceInfo dev;
   if (device_info(&dev) != TK_OK) return 0;
   return tk::plan_decode(desc->batch, desc->h_q, desc->h_kv, desc->r, desc->d_v,
-                         key_format(desc->k_dtype), dev->num_sms).bytes;
+                         key_format(desc->k_dtype), dev.num_sms).bytes;
 }
 
 namespace {
@@ -336,7 +341,8 @@ tk_status decode_impl(const tk_cache_desc* desc, const void* q, const void* k_ca
                       const void* v_cache, const float* k_scale, const int32_t* page_table,
                       const int32_t* seq_lens, const void* k_new, const void* v_new,
                       int32_t max_seq_len, void* out, int32_t out_dtype, float scale,
-                      void* workspace, size_t workspace_bytes, void* stream) {
+                      void* workspace, size_t workspace_bytes, bool clear_counters,
+                      void* stream) {
   const bool fuse = k_new != nullptr || v_new != nullptr;
   tk_status s = check_desc(desc);
   if (s != TK_OK) return s;
@@ -352,10 +358,10 @@ tk_status decode_impl(const tk_cache_desc* desc, const void* q, const void* k_ca
   if (fuse && (!k_new || !v_new)) return fail(TK_ERR_INVALID_ARG, "k_new / v_new is NULL");
   if (fuse && (!aligned16(k_new) || !aligned16(v_new)))
     return fail(TK_ERR_INVALID_ARG, "k_new / v_new must be 16-byte aligned");
-  DeviceInfo* dev;
+  DeviceInfo dev;
   if ((s = device_info(&dev)) != TK_OK) return s;
   const tk::DecodePlan pl = tk::plan_decode(desc->batch, desc->h_q, desc->h_kv, desc->r, desc->d_v,
-                                            key_format(desc->k_dtype), dev->num_sms);
+                                            key_format(desc->k_dtype), dev.num_sms);
   if (!workspace || (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
     return fail(TK_ERR_WORKSPACE, "workspace is NULL or not 256-byte aligned");
   if (workspace_bytes < pl.bytes)
@@ -366,7 +372,7 @@ tk_status decode_impl(const tk_cache_desc* desc, const void* q, const void* k_ca
   p.seq_lens = seq_lens; p.out = out; p.out_f32 = out_dtype == TK_F32;
   p.counters = reinterpret_cast<int32_t*>(ws + pl.off_counters);
   p.part = reinterpret_cast<float*>(ws + pl.off_part);
-  p.err = dev->err;
+  p.err = dev.err;
   p.B = desc->batch; p.Hq = desc->h_q; p.Hkv = desc->h_kv; p.R = desc->r; p.DV = desc->d_v;
   p.G = desc->h_q / desc->h_kv;
   p.k_fmt = key_format(desc->k_dtype);
@@ -380,6 +386,12 @@ tk_status decode_impl(const tk_cache_desc* desc, const void* q, const void* k_ca
   p.fuse_append = fuse;
   p.k_new = k_new;
   p.v_new = v_new;
+  if (clear_counters && tk::decode_max_batch() >= p.B) {
+    // every check has passed: zero the arrival counters right before the launch
+    const cudaError_t ce = cudaMemsetAsync(p.counters, 0, static_cast<size_t>(p.B) * p.Hkv * sizeof(int32_t),
+                                           static_cast<cudaStream_t>(stream));
+    if (ce != cudaSuccess) return cuda_fail(ce, "clear arrival counters");
+  }
   int uns = 0;
   cudaError_t e = tk::launch_decode(p, static_cast<cudaStream_t>(stream), &uns);
   if (uns) return fail(TK_ERR_UNSUPPORTED, "decode: no kernel for this shape (batch <= %d)",
@@ -395,7 +407,7 @@ tk_status tk_attn_decode(const tk_cache_desc* desc, const void* q, const void* k
                          int32_t out_dtype, float scale, void* workspace,
                          size_t workspace_bytes, void* stream) {
   return decode_impl(desc, q, k_cache, v_cache, k_scale, page_table, seq_lens, nullptr, nullptr,
-                     max_seq_len, out, out_dtype, scale, workspace, workspace_bytes, stream);
+                     max_seq_len, out, out_dtype, scale, workspace, workspace_bytes, false, stream);
 }
 
 tk_status tk_attn_decode_append(const tk_cache_desc* desc, const void* q, void* k_cache,
@@ -405,8 +417,26 @@ tk_status tk_attn_decode_append(const tk_cache_desc* desc, const void* q, void* 
                                 void* workspace, size_t workspace_bytes, void* stream) {
   if (!k_new || !v_new) return fail(TK_ERR_INVALID_ARG, "k_new / v_new is NULL");
   return decode_impl(desc, q, k_cache, v_cache, k_scale, page_table, seq_lens, k_new, v_new,
-                     max_seq_len, out, out_dtype, scale, workspace, workspace_bytes, stream);
+                     max_seq_len, out, out_dtype, scale, workspace, workspace_bytes, false, stream);
 }
+
+}  // extern "C"
+
+namespace tk {
+// tk_attn_decode on a caller-supplied scratch whose arrival counters are
+// cleared in stream order once every argument check has passed (used by
+// tk_attn_decode_noalloc, whose scratch other calls may have left dirty).
+tk_status decode_on_scratch(const tk_cache_desc* desc, const void* q, const void* k_cache,
+                            const void* v_cache, const float* k_scale, const int32_t* page_table,
+                            const int32_t* seq_lens, int32_t max_seq_len, void* out,
+                            int32_t out_dtype, float scale, void* scratch, size_t scratch_bytes,
+                            void* stream) {
+  return decode_impl(desc, q, k_cache, v_cache, k_scale, page_table, seq_lens, nullptr, nullptr,
+                     max_seq_len, out, out_dtype, scale, scratch, scratch_bytes, true, stream);
+}
+}  // namespace tk
+
+extern "C" {
 
 tk_status tk_copy_async(void* dst, const void* src, size_t bytes, void* stream) {
   if (bytes == 0) return TK_OK;
@@ -416,20 +446,32 @@ tk_status tk_copy_async(void* dst, const void* src, size_t bytes, void* stream) 
   return TK_OK;
 }
 
+tk_status tk_check_wait_timeout(int32_t limit_us, void* stream) {
+  if (limit_us < 1 || limit_us > 1000000)
+    return fail(TK_ERR_INVALID_ARG, "limit_us=%d (1 .. 1000000)", limit_us);
+  DeviceInfo dev;
+  tk_status s = device_info(&dev);
+  if (s != TK_OK) return s;
+  const cudaError_t e = tk::launch_wait_timeout(dev.err, static_cast<uint64_t>(limit_us) * 1000u,
+                                                static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "wait-timeout check launch");
+  return TK_OK;
+}
+
 tk_status tk_get_device_error(int32_t* code_out, void* stream) {
   if (!code_out) return fail(TK_ERR_INVALID_ARG, "code_out is NULL");
-  DeviceInfo* dev;
+  DeviceInfo dev;
   tk_status s = device_info(&dev);
   if (s != TK_OK) return s;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   cudaError_t e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
   int v = 0;
-  e = cudaMemcpy(&v, dev->err, sizeof(int), cudaMemcpyDeviceToHost);
+  e = cudaMemcpy(&v, dev.err, sizeof(int), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return cuda_fail(e, "read device error word");
   if (v != 0) {
     const int zero = 0;
-    e = cudaMemcpy(dev->err, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    e = cudaMemcpy(dev.err, &zero, sizeof(int), cudaMemcpyHostToDevice);
     if (e != cudaSuccess) return cuda_fail(e, "clear device error word");
   }
   *code_out = v;

@@ -184,3 +184,10 @@ def test_host_output_needs_page_locked_memory():
         tb._need_out(torch.empty(4, 8), "out", None)          # pageable host memory
     with pytest.raises(TypeError):
         tb._need_out(torch.empty(4, 8, dtype=torch.float16), "out", None)
+
+
+def test_wait_timeout_check_validation(lib):
+    """tk_check_wait_timeout rejects a limit outside 1 us .. 1 s before any CUDA call."""
+    assert lib.tk_check_wait_timeout(0, None) == tb.TK_ERR_INVALID_ARG
+    assert "limit_us" in tb.tk_last_error()
+    assert lib.tk_check_wait_timeout(1000001, None) == tb.TK_ERR_INVALID_ARG

@@ -3,8 +3,8 @@
 The append must store exactly the oracle's packed codes and scales; decode
 must match the fp64 oracle on the dequantised keys for every (r >= 32, d_v,
 G), give identical bits for paged and contiguous caches, and the fused
-append + decode must equal the two calls.  The full-size int8-workload shape
-(B=64, context 32768) is checked on sampled heads.
+append + decode must equal the two calls.  The full-size shape (B=64,
+context 32768) at every r is in test_gpu_fullsize.py.
 """
 
 import math
@@ -120,23 +120,3 @@ def test_int4_fused_append_decode_equals_two_calls():
     assert tb.tk_get_device_error() == 0
     assert torch.equal(out_a, out_f)
     assert torch.equal(a.k, f.k) and torch.equal(a.k_scale, f.k_scale) and torch.equal(a.v, f.v)
-
-
-def test_int4_decode_full_size_sampled():
-    """B=64, H_q=32, H_kv=8, r=32, d_v=128, context 32768, int4 keys: sampled heads."""
-    require_gpu()
-    B, hq, hkv, r, dv, L = 64, 32, 8, 32, 128, 32768
-    cache, kn, _ = _filled(B, hq, hkv, r, dv, L, seed=1021)
-    q = inputs.normal_bf16((B, hq, r), seed=1022, device="cuda")
-    out = _run(cache, q, [L] * B)
-    rng = np.random.default_rng(2)
-    got, ref = [], []
-    for b in rng.choice(B, 6, replace=False):
-        for h in rng.choice(hq, 2, replace=False):
-            g = h // (hq // hkv)
-            codes, sc = oc.quantize_int4_per_token(kn[b, g].float().cpu().numpy())
-            assert np.array_equal(cache.k[b, g].cpu().numpy(), oc.pack_int4(codes))
-            kk = oa.dequantize_keys(codes, sc)
-            ref.append(oa.attention_head(f64(q[b, h])[None], kk, f64(cache.v[b, g]), 1 / math.sqrt(r))[0])
-            got.append(f64(out[b, h]))
-    parity(np.stack(got), np.stack(ref), what="int4 full size")

@@ -33,28 +33,51 @@ def _cache(B, hq, hkv, r, dv, lens, k_int8, seed):
     return cache
 
 
-@pytest.mark.parametrize("shape", [
+SHAPES = {
     # Mistral-7B-shaped GQA decode, every context 4096
-    dict(B=16, hq=32, hkv=8, r=32, dv=128, lens=[4096] * 16, k_int8=False),
+    "mistral": dict(B=16, hq=32, hkv=8, r=32, dv=128, lens=[4096] * 16, k_int8=False),
     # ragged contexts, int8 keys, including an empty and a one-token context
-    dict(B=4, hq=16, hkv=4, r=64, dv=64, lens=[3000, 0, 1, 1234], k_int8=True),
-])
-def test_noalloc_matches_workspace_decode_twice(shape):
-    require_gpu()
-    s = shape
-    cache = _cache(s["B"], s["hq"], s["hkv"], s["r"], s["dv"], s["lens"], s["k_int8"], seed=77)
-    q = inputs.normal_bf16((s["B"], s["hq"], s["r"]), 78, device="cuda")
+    "ragged_int8": dict(B=4, hq=16, hkv=4, r=64, dv=64, lens=[3000, 0, 1, 1234], k_int8=True),
+}
+
+
+def _case(name, seed):
+    s = SHAPES[name]
+    cache = _cache(s["B"], s["hq"], s["hkv"], s["r"], s["dv"], s["lens"], s["k_int8"], seed=seed)
+    q = inputs.normal_bf16((s["B"], s["hq"], s["r"]), seed + 1, device="cuda")
     sl = torch.tensor(s["lens"], dtype=torch.int32, device="cuda")
     L = max(s["lens"])
     assert tb.tk_decode_workspace_size(cache.desc, L) <= 8 << 20
+    # the regular entry point, with a workspace of its own, zero-filled
     ref = torch.empty(s["B"], s["hq"], s["dv"], device="cuda")
     tb.tk_attn_decode(cache, q, sl, L, ref, tb.decode_workspace(cache.desc, L))
+    return cache, q, sl, L, ref
+
+
+@pytest.mark.parametrize("name", sorted(SHAPES))
+def test_noalloc_matches_workspace_decode_twice(name):
+    require_gpu()
+    cache, q, sl, L, ref = _case(name, seed=77)
     for _ in range(2):
         out = torch.full_like(ref, float("nan"))
         tb.tk_attn_decode_noalloc(cache, q, sl, L, out)
         assert tb.tk_get_device_error() == 0
         parity(f64(out), f64(ref), what="noalloc vs workspace decode")
         assert torch.equal(out, ref)  # same kernel and split plan: identical bits
+
+
+def test_noalloc_alternating_shapes():
+    """Calls of different shapes in a row: each finds the scratch as a call of
+    the other shape (another batch x h_kv, other partial records) left it."""
+    require_gpu()
+    cases = {n: _case(n, seed=91 + 10 * i) for i, n in enumerate(("mistral", "ragged_int8"))}
+    for name in ("mistral", "ragged_int8", "mistral", "ragged_int8"):
+        cache, q, sl, L, ref = cases[name]
+        out = torch.full_like(ref, float("nan"))
+        tb.tk_attn_decode_noalloc(cache, q, sl, L, out)
+        assert tb.tk_get_device_error() == 0
+        parity(f64(out), f64(ref), what=f"noalloc {name} after another shape")
+        assert torch.equal(out, ref)
 
 
 def test_noalloc_rejects_shapes_beyond_its_scratch():
