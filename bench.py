@@ -369,14 +369,16 @@ def measure_prefill(w, iters, device, torch):
     return {"ms": sec * 1e3, "tflops": flops / sec / 1e12, "flops_per_launch": flops}
 
 
-def measure_chunked_prefill(w, iters, device, torch):
+def measure_chunked_prefill(w, iters, device, torch, k_fmt="bf16"):
     """A prompt chunk of w.seq tokens after w.cached cached ones: tk_attn_prefill_cached
-    (append of the chunk + attention over the cache), bf16 output."""
+    (append of the chunk + attention over the cache), bf16 output; keys stored as
+    bf16, int8 or int4.  The append launch is also timed on its own."""
     from paper_2603_04427_gb300 import binding as tb
     from paper_2603_04427_gb300 import cost_model as cm
     from paper_2603_04427_gb300 import inputs
     B, hq, hkv, S, r, dv, L0 = w.batch, w.h_q, w.h_kv, w.seq, w.r, w.d_v, w.cached
-    cache = tb.ThinKeyCache.allocate(B, hq, hkv, r, dv, capacity=L0 + S, device=device)
+    cache = tb.ThinKeyCache.allocate(B, hq, hkv, r, dv, capacity=L0 + S, device=device,
+                                     k_int8=k_fmt == "int8", k_int4=k_fmt == "int4")
     zero = torch.zeros(B, dtype=torch.int32, device=device)
     tb.tk_kv_append(cache, inputs.normal_bf16((B, hkv, L0, r), w.seed + 1, device=device),
                     inputs.normal_bf16((B, hkv, L0, dv), w.seed + 2, device=device), zero)
@@ -389,10 +391,14 @@ def measure_chunked_prefill(w, iters, device, torch):
     def enq(_):  # the same chunk re-appended at the same positions every time
         tb.tk_attn_prefill_cached(cache, q, kn, vn, sl, L0 + S, out)
 
+    def enq_append(_):
+        tb.tk_kv_append(cache, kn, vn, sl)
+
     sec = graph_time(torch, enq, iters, 3, max_graph=16, min_seconds=0.3) / iters
+    sec_app = graph_time(torch, enq_append, iters, 3, max_graph=16, min_seconds=0.1) / iters
     flops = cm.prefill_flops(B, hq, S, r, dv, cached=L0)
     return {"ms": sec * 1e3, "tflops": flops / sec / 1e12, "flops_per_call": flops,
-            "cached": L0, "launches": 2}
+            "cached": L0, "launches": 2, "append_ms": sec_app * 1e3, "k_dtype": k_fmt}
 
 
 def measure_backward(w, iters, device, torch):
@@ -746,7 +752,8 @@ def main():
         elif args.only == "backward":
             res.update(measure_backward(wl.MHA7B_PREFILL, args.steps, device, torch))
         elif args.only == "chunked":
-            res.update(measure_chunked_prefill(wl.CHUNKED_PREFILL, args.steps, device, torch))
+            for kf in ("bf16", "int8", "int4"):
+                res[kf] = measure_chunked_prefill(wl.CHUNKED_PREFILL, args.steps, device, torch, k_fmt=kf)
         elif args.only == "gpt2":
             res.update(measure_gpt2_layer(wl.GPT2_LAYER, args.steps, device, torch))
         else:
@@ -868,10 +875,13 @@ def main():
             tflops=r3(bw["tflops"]), frac=r3(bw["tflops"] / peaks["bf16_tflops"]),
             flops_per_call=bw["flops_per_call"], launches=bw["launches"])
         cw = wl.CHUNKED_PREFILL
-        cp = measure_chunked_prefill(cw, 20, device, torch)
-        extra[cw.name] = dict(cw.as_config(), ms=r3(cp["ms"]), tflops=r3(cp["tflops"]),
-                              frac=r3(cp["tflops"] / peaks["bf16_tflops"]),
-                              flops_per_call=cp["flops_per_call"], launches=cp["launches"])
+        for kf in ("bf16", "int8"):
+            cp = measure_chunked_prefill(cw, 20, device, torch, k_fmt=kf)
+            name = cw.name if kf == "bf16" else cw.name + "_int8_keys"
+            extra[name] = dict(cw.as_config(), k_dtype=kf, ms=r3(cp["ms"]), tflops=r3(cp["tflops"]),
+                               frac=r3(cp["tflops"] / peaks["bf16_tflops"]),
+                               append_ms=r3(cp["append_ms"]), flops_per_call=cp["flops_per_call"],
+                               launches=cp["launches"])
         line["workloads"] = extra
         # the causal prefill half of the metric, last on the line
         pf = measure_prefill(pw, 20, device, torch)
@@ -889,7 +899,8 @@ def main():
         if n == 1:
             try:
                 procs = host_cores()
-                cal = cpu_oracle_prefill(pw, 512, 1, 1)
+                # calibrate on the same blocks (the last one, near row S, is the slowest)
+                cal = cpu_oracle_prefill(pw, 512, 1, procs, warmup=0)
                 reps = max(1, int(10.0 / cal["sec"]))
                 cb = cpu_oracle_prefill(pw, 512, reps, procs)
                 pre["cpu_baseline"] = {k: (r3(v) if isinstance(v, float) else v) for k, v in cb.items()}

@@ -58,7 +58,7 @@
 extern "C" {
 #endif
 
-#define TK_ABI_VERSION 1
+#define TK_ABI_VERSION 2
 
 typedef enum tk_status {
   TK_OK = 0,
@@ -188,25 +188,30 @@ tk_status tk_attn_backward(const void* q, const void* k, const void* v, const vo
 /* Prefill of a chunk of `seq` new tokens per sequence against the cache
  * (Section 2.1, Eqs. 1-4, over a context that continues an existing one):
  * first writes the chunk's thin keys and values at positions
- * seq_lens[b] .. seq_lens[b] + seq - 1 exactly as tk_kv_append, then
- * computes, for query i of the chunk (position seq_lens[b] + i),
- * attention over the cache's tokens 0 .. seq_lens[b] + i (causal, aligned
- * to the end of the context) or over all seq_lens[b] + seq of them
- * (causal == 0).
+ * seq_lens[b] .. seq_lens[b] + seq - 1 exactly as tk_kv_append (int8 / int4
+ * keys quantised the same way, bit for bit), then computes, for query i of
+ * the chunk (position seq_lens[b] + i), attention over the cache's tokens
+ * 0 .. seq_lens[b] + i (causal, aligned to the end of the context) or over
+ * all seq_lens[b] + seq of them (causal == 0).
  *   q        : device bf16 [batch][h_q][seq][r]       the chunk's queries
+ *   k_scale  : device fp32 per-token key scales (int8 / int4 keys, else NULL)
  *   k_new    : device bf16 [batch][h_kv][seq][r]      the chunk's thin keys
  *   v_new    : device bf16 [batch][h_kv][seq][d_v]    the chunk's values
  *   seq_lens : device int32 [batch], tokens cached before the chunk (not
  *              modified; the caller advances it by seq afterwards)
  *   max_seq_len: host bound of seq_lens[b] + seq
  *   out      : device [batch][h_q][seq][d_v], TK_BF16 or TK_F32
- * bf16 keys only (TK_ERR_UNSUPPORTED otherwise): the products run on the
- * tensor cores from bf16 tiles.  Contiguous or paged caches; a sequence whose
- * chunk does not fit sets the device error word and is computed over a
- * clamped context.  seq_lens[b] == 0 gives the plain causal prefill of the
- * chunk.  Two launches (append, then attention) in stream order.           */
+ * Keys of every k_dtype (Section 6: thin keys compose with key
+ * quantisation): the products run on the tensor cores from bf16 tiles, int8
+ * and int4 codes widened to bf16 exactly in shared memory, and each score
+ * q . code multiplied by its key's fp32 scale.  Contiguous or paged caches;
+ * a sequence whose chunk does not fit sets the device error word and is
+ * computed over a clamped context.  Cache slots past a sequence's context
+ * may hold anything (they are never weighted).  seq_lens[b] == 0 gives the
+ * plain causal prefill of the chunk.  Two launches (append, then attention)
+ * in stream order.                                                        */
 tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void* k_cache,
-                                 void* v_cache, const int32_t* page_table,
+                                 void* v_cache, float* k_scale, const int32_t* page_table,
                                  const int32_t* seq_lens, const void* k_new, const void* v_new,
                                  int32_t seq, int32_t max_seq_len, void* out, int32_t out_dtype,
                                  float scale, int32_t causal, void* stream);

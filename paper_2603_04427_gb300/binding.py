@@ -63,8 +63,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tk_backward_workspace_size": (sz, [i32, i32, i32]),
         "tk_attn_backward": (i32, [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, i32, i32, i32, i32,
                                    i32, i32, f32, i32, vp]),
-        "tk_attn_prefill_cached": (i32, [dp, vp, vp, vp, vp, vp, vp, vp, i32, i32, vp, i32, f32,
-                                         i32, vp]),
+        "tk_attn_prefill_cached": (i32, [dp, vp, vp, vp, vp, vp, vp, vp, vp, i32, i32, vp, i32,
+                                         f32, i32, vp]),
         "tk_attn_decode": (i32, [dp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp, sz, vp]),
         "tk_attn_decode_append": (i32, [dp, vp, vp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp,
                                         sz, vp]),
@@ -314,7 +314,7 @@ def tk_attn_prefill_cached(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_s
                            scale: float | None = None, causal: bool = True, stream=None):
     """Append a chunk (k_new [B, H_kv, S, r], v_new [B, H_kv, S, d_v] bf16) at seq_lens[b]
     and prefill its queries q [B, H_q, S, r] over the cache (query i at position
-    seq_lens[b] + i) -> out [B, H_q, S, d_v] (fp32 or bf16)."""
+    seq_lens[b] + i) -> out [B, H_q, S, d_v] (fp32 or bf16).  bf16, int8 or int4 keys."""
     d = cache.desc
     dev = cache.k.device
     for t, n in ((q, "q"), (k_new, "k_new"), (v_new, "v_new")):
@@ -331,7 +331,8 @@ def tk_attn_prefill_cached(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_s
     scale = 1.0 / math.sqrt(d.r) if scale is None else float(scale)
     L = load_library()
     _check(L.tk_attn_prefill_cached(ctypes.byref(d), _ptr(q), _ptr(cache.k), _ptr(cache.v),
-                                    _ptr(cache.page_table), _ptr(seq_lens), _ptr(k_new), _ptr(v_new),
+                                    _ptr(cache.k_scale), _ptr(cache.page_table), _ptr(seq_lens),
+                                    _ptr(k_new), _ptr(v_new),
                                     S, int(max_seq_len), _ptr(out),
                                     TK_F32 if out.dtype == torch.float32 else TK_BF16, scale,
                                     1 if causal else 0, _stream(stream)), "tk_attn_prefill_cached")

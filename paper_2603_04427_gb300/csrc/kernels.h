@@ -100,6 +100,8 @@ struct PrefillParams {
   int capacity;             // contiguous cache rows per (b, g)
   int page_size, page_shift, num_pages, max_pages;  // paged (page_size 0 = contiguous)
   int kv_limit;             // bound of seq_lens[b] + S
+  int k_fmt;                // cache keys: 0 bf16, 1 int8, 2 int4 (cached mode only)
+  const float* k_scale;     // fp32 per-token key scales (int8 / int4 keys)
   float* lse;               // optional [B][Hq][S]: natural-log logsumexp of each row's scores
 };
 

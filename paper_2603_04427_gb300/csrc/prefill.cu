@@ -71,7 +71,10 @@ __device__ __forceinline__ float max128(const uint32_t* v) {
 }
 
 
-template <int R, int DV>
+// Key formats of the cache a chunked prefill reads (the plain prefill is always bf16).
+constexpr int kKeyBF16 = 0, kKeyInt8 = 1, kKeyInt4 = 2;
+
+template <int R, int DV, int KF = kKeyBF16>
 struct PCfg {
   // Q / K rows are r bf16 = 2r bytes: swizzle span = min(2r, 128) bytes; a row
   // wider than 128 bytes is loaded as 128-byte-wide boxes.
@@ -86,18 +89,64 @@ struct PCfg {
   static constexpr int VB = kBN * DV * 2;
   static constexpr int V_NBOX = DV / 64;             // 128-byte-wide boxes of V
   static constexpr int V_BOXB = kBN * 128;
+  // quantised keys: a tile's codes (r or r/2 bytes per key) land in a staging
+  // area of the stage, and its 128 fp32 key scales after them
+  static constexpr int CODE_ROWB = KF == kKeyInt8 ? R : (KF == kKeyInt4 ? R / 2 : 0);
+  static constexpr int STGB = kBN * CODE_ROWB;
+  static constexpr int SCB = KF == kKeyBF16 ? 0 : kBN * 4;
   static constexpr int QBA = (QB + 1023) / 1024 * 1024;  // one Q tile, 1 KB aligned
   static constexpr int OFF_Q = 0;                        // two Q tiles
   static constexpr int OFF_K = 2 * QBA;
   static constexpr int KBA = (KB + 1023) / 1024 * 1024;
   static constexpr int STAGE = KBA + VB;
-  static constexpr int NST = (2 * QBA + 3 * STAGE + 2048 <= 200 * 1024) ? 3 : 2;
-  static constexpr int OFF_BAR = OFF_K + NST * STAGE;
+  static constexpr int NST = (2 * QBA + 3 * (STAGE + SCB) + STGB + 2048 <= 200 * 1024) ? 3 : 2;
+  // one staging area serves every stage (the TMA warp widens a tile's codes
+  // before it loads the next tile's); the scales keep one slot per stage
+  static constexpr int OFF_STG = OFF_K + NST * STAGE;
+  static constexpr int OFF_SC = OFF_STG + STGB;
+  static constexpr int OFF_BAR = OFF_SC + NST * SCB;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;      // + slack to align the base to 1 KB
   static_assert(SMEM <= 227 * 1024, "shared memory");
   static constexpr uint32_t IDESC_S = instr_desc(kBM, kBN, false);
   static constexpr uint32_t IDESC_O = instr_desc(kBM, DV, true);
 };
+
+// Byte offset, inside a K tile, of the 16-byte piece holding elements e0 .. e0+7
+// (e0 a multiple of 8) of key `row`, in the layout the TMA writes with the
+// tile's swizzle: box e0 / QK_BOX, row pitch QK_SW bytes, and the piece's index
+// within its row XORed with address bits 7.. (32-, 64- or 128-byte swizzle).
+template <class C>
+__device__ __forceinline__ uint32_t k_piece_offset(int row, int e0) {
+  const uint32_t o = static_cast<uint32_t>(row * C::QK_SW + (e0 % C::QK_BOX) * 2);
+  constexpr uint32_t mask = static_cast<uint32_t>(C::QK_SW / 16 - 1) << 4;
+  return static_cast<uint32_t>((e0 / C::QK_BOX) * C::QK_BOXB) + (o ^ ((o >> 3) & mask));
+}
+
+// Four int8 codes (one per byte) -> two words of two bf16 each (element 4i in the
+// low half of the first word); exact: |code| <= 127 is a bf16 value.
+__device__ __forceinline__ uint2 int8x4_to_bf16(uint32_t w) {
+  float f[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    f[i] = static_cast<float>(static_cast<int>(static_cast<int8_t>((w >> (8 * i)) & 0xffu)));
+  __nv_bfloat162 a = __floats2bfloat162_rn(f[0], f[1]), b = __floats2bfloat162_rn(f[2], f[3]);
+  return make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&b));
+}
+
+// Two bytes of packed int4 codes (element 2j in the low nibble of byte j, 2j+1 in
+// the high nibble, 4-bit two's complement) -> two words of two bf16 each; exact.
+__device__ __forceinline__ uint2 int4x4_to_bf16(uint32_t two_bytes) {
+  int c[4];
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int b = static_cast<int>((two_bytes >> (8 * i)) & 0xffu);
+    c[2 * i] = static_cast<int>(static_cast<int8_t>(b << 4)) >> 4;
+    c[2 * i + 1] = static_cast<int>(static_cast<int8_t>(b)) >> 4;
+  }
+  __nv_bfloat162 a = __floats2bfloat162_rn(static_cast<float>(c[0]), static_cast<float>(c[1]));
+  __nv_bfloat162 d = __floats2bfloat162_rn(static_cast<float>(c[2]), static_cast<float>(c[3]));
+  return make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&d));
+}
 
 struct Maps {
   CUtensorMap q, k, v;
@@ -114,10 +163,10 @@ struct Maps {
 //   warps 4-7: the same for tile B
 //   warp 8: TMA producer (Q tiles once, K/V tiles into an NST-stage ring)
 //   warp 9: MMA issuer
-template <int R, int DV>
+template <int R, int DV, int KF>
 __global__ void __launch_bounds__(kThreads, 1)
 prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
-  using C = PCfg<R, DV>;
+  using C = PCfg<R, DV, KF>;
   constexpr int NST = C::NST;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
@@ -130,7 +179,8 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   uint64_t* s_full = kv_empty + NST;            // [2] (tile A, tile B)
   uint64_t* p_full = s_full + 2;                // [tile][part]: P of one key range
   uint64_t* o_full = p_full + 2 * kParts;       // [2]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_full + 2);
+  uint64_t* c_full = o_full + 2;                // [NST] cached mode: raw K tile (+ scales) landed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(c_full + NST);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int n_qt = (p.S + kBM - 1) / kBM;
@@ -173,6 +223,7 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       mbar_init(&k_full[s], 1);
       mbar_init(&v_full[s], 1);
       mbar_init(&kv_empty[s], 1);
+      mbar_init(&c_full[s], 1);
     }
     for (int x = 0; x < 2; ++x) {
       mbar_init(&s_full[x], 1);
@@ -197,6 +248,7 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
     const int g = h / (p.Hq / p.Hkv);
     const int bps = (p.page_size == 0 || p.page_size >= kBN) ? kBN : p.page_size;
     const int nsub = kBN / bps;
+    const bool relay = p.seq_lens != nullptr;   // cached mode: K tiles pass through this warp
     if (lane == 0) {
       prefetch_map(&maps.q);
       prefetch_map(&maps.k);
@@ -233,19 +285,93 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
         planes[s2] = __shfl_sync(0xffffffffu, plane, s2);
         rows[s2] = __shfl_sync(0xffffffffu, row, s2);
       }
+      unsigned char* sk = smem + C::OFF_K + st * C::STAGE;
+      unsigned char* sv = sk + C::KBA;
       if (lane == 0) {
-        unsigned char* sk = smem + C::OFF_K + st * C::STAGE;
-        unsigned char* sv = sk + C::KBA;
-        mbar_arrive_expect_tx(&k_full[st], C::KB);
-        for (int s2 = 0; s2 < nsub; ++s2)
-          for (int i = 0; i < C::QK_NBOX; ++i)
-            tma_load_3d(sk + i * C::QK_BOXB + s2 * bps * C::QK_SW, &maps.k, i * C::QK_BOX,
-                        rows[s2], planes[s2], &k_full[st]);
+        if (!relay) {
+          mbar_arrive_expect_tx(&k_full[st], C::KB);
+          for (int s2 = 0; s2 < nsub; ++s2)
+            for (int i = 0; i < C::QK_NBOX; ++i)
+              tma_load_3d(sk + i * C::QK_BOXB + s2 * bps * C::QK_SW, &maps.k, i * C::QK_BOX,
+                          rows[s2], planes[s2], &k_full[st]);
+        } else if constexpr (KF == kKeyBF16) {
+          mbar_arrive_expect_tx(&c_full[st], C::KB);
+          for (int s2 = 0; s2 < nsub; ++s2)
+            for (int i = 0; i < C::QK_NBOX; ++i)
+              tma_load_3d(sk + i * C::QK_BOXB + s2 * bps * C::QK_SW, &maps.k, i * C::QK_BOX,
+                          rows[s2], planes[s2], &c_full[st]);
+        } else {
+          // raw codes into the staging area, the tile's key scales after them
+          unsigned char* stg = smem + C::OFF_STG;
+          float* sc = reinterpret_cast<float*>(smem + C::OFF_SC + st * C::SCB);
+          const int kv0 = j * kBN;
+          uint32_t sc_bytes = 0;
+          if (p.page_size == 0) {
+            sc_bytes = static_cast<uint32_t>(min(kBN, p.capacity - kv0)) * 4u;
+          } else {
+            for (int s2 = 0; s2 < nsub; ++s2)
+              if (planes[s2] >= 0) sc_bytes += static_cast<uint32_t>(bps) * 4u;
+          }
+          mbar_arrive_expect_tx(&c_full[st], static_cast<uint32_t>(nsub * bps * C::CODE_ROWB) + sc_bytes);
+          for (int s2 = 0; s2 < nsub; ++s2)
+            tma_load_3d(stg + s2 * bps * C::CODE_ROWB, &maps.k, 0, rows[s2], planes[s2], &c_full[st]);
+          if (p.page_size == 0) {
+            bulk_g2s(sc, p.k_scale + static_cast<size_t>(kv_plane) * p.capacity + kv0, sc_bytes,
+                     &c_full[st]);
+          } else {
+            for (int s2 = 0; s2 < nsub; ++s2)
+              if (planes[s2] >= 0)
+                bulk_g2s(sc + s2 * bps,
+                         p.k_scale + static_cast<size_t>(planes[s2]) * p.page_size + rows[s2],
+                         static_cast<uint32_t>(bps) * 4u, &c_full[st]);
+          }
+        }
         mbar_arrive_expect_tx(&v_full[st], C::VB);
         for (int s2 = 0; s2 < nsub; ++s2)
           for (int i = 0; i < C::V_NBOX; ++i)
             tma_load_3d(sv + i * C::V_BOXB + s2 * bps * 128, &maps.v, i * 64, rows[s2], planes[s2],
                         &v_full[st]);
+      }
+      if (relay) {
+        // Cached mode: the warp finishes the K tile before the MMA warp may read
+        // it -- quantised codes are widened to bf16 in the tile's swizzled layout,
+        // and on the tile that holds the context's end the value rows past it are
+        // zeroed (the cache may hold anything there, and 0 * NaN would spread).
+        const uint32_t ph = (j / NST) & 1;
+        bool okc = mbar_wait(&c_full[st], ph, p.err);
+        const int kv0 = j * kBN, n_valid = kv_len - kv0;
+        if (n_valid < kBN) okc = mbar_wait(&v_full[st], ph, p.err) && okc;
+        if (!__all_sync(0xffffffffu, okc)) break;
+        if constexpr (KF != kKeyBF16) {
+          const unsigned char* stg = smem + C::OFF_STG;
+          constexpr int PPR = R / 8;  // 16-byte bf16 pieces per key row
+#pragma unroll 4
+          for (int c = lane; c < kBN * PPR; c += 32) {
+            const int row = c / PPR, e0 = (c % PPR) * 8;
+            uint2 lo, hi;
+            if constexpr (KF == kKeyInt8) {
+              const uint2 w = *reinterpret_cast<const uint2*>(stg + row * C::CODE_ROWB + e0);
+              lo = int8x4_to_bf16(w.x);
+              hi = int8x4_to_bf16(w.y);
+            } else {
+              const uint32_t w = *reinterpret_cast<const uint32_t*>(stg + row * C::CODE_ROWB + e0 / 2);
+              lo = int4x4_to_bf16(w & 0xffffu);
+              hi = int4x4_to_bf16(w >> 16);
+            }
+            *reinterpret_cast<uint4*>(sk + k_piece_offset<C>(row, e0)) = make_uint4(lo.x, lo.y, hi.x, hi.y);
+          }
+        }
+        if (n_valid < kBN) {
+          const int first = max(n_valid, 0);
+          for (int c = lane; c < (kBN - first) * 8 * C::V_NBOX; c += 32) {
+            const int box = c / ((kBN - first) * 8), rem2 = c % ((kBN - first) * 8);
+            *reinterpret_cast<uint4*>(sv + box * C::V_BOXB + (first + rem2 / 8) * 128 + (rem2 % 8) * 16) =
+                make_uint4(0u, 0u, 0u, 0u);
+          }
+        }
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&k_full[st]);
       }
     }
   } else if (warp == 9) {
@@ -332,6 +458,21 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       // the whole S row of this thread: 128 fp32 scores
       uint32_t v[128];
       tmem_ld128(tS + lane_off, v);
+      if constexpr (KF != kKeyBF16) {
+        // quantised keys: the products are q . code; each key's fp32 scale turns
+        // them into q . k (the scales arrived with the codes on c_full)
+        const int st = j % NST;
+        if (!__all_sync(0xffffffffu, mbar_wait(&c_full[st], (j / NST) & 1, p.err))) { ok = false; break; }
+        const float4* sc4 = reinterpret_cast<const float4*>(smem + C::OFF_SC + st * C::SCB);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float4 f = sc4[i];
+          v[4 * i] = __float_as_uint(__uint_as_float(v[4 * i]) * f.x);
+          v[4 * i + 1] = __float_as_uint(__uint_as_float(v[4 * i + 1]) * f.y);
+          v[4 * i + 2] = __float_as_uint(__uint_as_float(v[4 * i + 2]) * f.z);
+          v[4 * i + 3] = __float_as_uint(__uint_as_float(v[4 * i + 3]) * f.w);
+        }
+      }
       if (masked) {
 #pragma unroll
         for (int i = 0; i < 128; ++i)
@@ -432,9 +573,9 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
 
 // ---------------------------------------------------------------- host side
 
-template <int R, int DV>
+template <int R, int DV, int KF>
 cudaError_t launch_t(const PrefillParams& p, cudaStream_t stream) {
-  using C = PCfg<R, DV>;
+  using C = PCfg<R, DV, KF>;
   Maps maps;
   // K / V: [B*Hkv][S] inputs, a contiguous cache [B*Hkv][capacity] or a paged
   // pool [num_pages*Hkv][page_size] (boxes of min(page_size, 128) rows)
@@ -446,11 +587,14 @@ cudaError_t launch_t(const PrefillParams& p, cudaStream_t stream) {
     kv_planes = p.num_pages * p.Hkv;
     box_rows = std::min(p.page_size, kBN);
   }
-  if (!make_map(&maps.q, p.q, R, p.S, p.B * p.Hq, C::QK_BOX, kBM, C::QK_SW) ||
-      !make_map(&maps.k, p.k, R, kv_rows, kv_planes, C::QK_BOX, box_rows, C::QK_SW) ||
-      !make_map(&maps.v, p.v, DV, kv_rows, kv_planes, 64, box_rows, 128))
-    return cudaErrorInvalidValue;
-  auto kern = prefill_kernel<R, DV>;
+  bool ok = make_map(&maps.q, p.q, R, p.S, p.B * p.Hq, C::QK_BOX, kBM, C::QK_SW) &&
+            make_map(&maps.v, p.v, DV, kv_rows, kv_planes, 64, box_rows, 128);
+  if constexpr (KF == kKeyBF16)
+    ok = ok && make_map(&maps.k, p.k, R, kv_rows, kv_planes, C::QK_BOX, box_rows, C::QK_SW);
+  else  // rows of codes, copied as they are into the staging area
+    ok = ok && make_map_bytes(&maps.k, p.k, C::CODE_ROWB, kv_rows, kv_planes, box_rows);
+  if (!ok) return cudaErrorInvalidValue;
+  auto kern = prefill_kernel<R, DV, KF>;
   const int smem = C::SMEM;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
@@ -465,11 +609,27 @@ cudaError_t launch_t(const PrefillParams& p, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
+template <int R, int DV>
+cudaError_t by_kf(const PrefillParams& p, cudaStream_t s, int* uns) {
+  // quantised keys only in cached mode (a cache written by the quantising append)
+  if (p.k_fmt == kKeyBF16) return launch_t<R, DV, kKeyBF16>(p, s);
+  if (!p.seq_lens || !p.k_scale) {
+    *uns = 1;
+    return cudaSuccess;
+  }
+  if (p.k_fmt == kKeyInt8) return launch_t<R, DV, kKeyInt8>(p, s);
+  if constexpr (R >= 32) {
+    if (p.k_fmt == kKeyInt4) return launch_t<R, DV, kKeyInt4>(p, s);
+  }
+  *uns = 1;
+  return cudaSuccess;
+}
+
 template <int R>
 cudaError_t by_dv(const PrefillParams& p, cudaStream_t s, int* uns) {
   switch (p.DV) {
-    case 64: return launch_t<R, 64>(p, s);
-    case 128: return launch_t<R, 128>(p, s);
+    case 64: return by_kf<R, 64>(p, s, uns);
+    case 128: return by_kf<R, 128>(p, s, uns);
   }
   *uns = 1;
   return cudaSuccess;

@@ -263,15 +263,12 @@ tk_status prefill_impl(const void* q, const void* k, const void* v, void* out, f
 }  // namespace
 
 tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void* k_cache,
-                                 void* v_cache, const int32_t* page_table,
+                                 void* v_cache, float* k_scale, const int32_t* page_table,
                                  const int32_t* seq_lens, const void* k_new, const void* v_new,
                                  int32_t seq, int32_t max_seq_len, void* out, int32_t out_dtype,
                                  float scale, int32_t causal, void* stream) {
   tk_status s = check_desc(desc);
   if (s != TK_OK) return s;
-  if (desc->k_dtype != TK_BF16)
-    return fail(TK_ERR_UNSUPPORTED, "prefill over a cache needs bf16 keys (k_dtype=%d)",
-                desc->k_dtype);
   if (seq < 0 || max_seq_len < seq)
     return fail(TK_ERR_INVALID_ARG, "seq=%d max_seq_len=%d", seq, max_seq_len);
   if (out_dtype != TK_BF16 && out_dtype != TK_F32)
@@ -279,7 +276,7 @@ tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void*
   if (!std::isfinite(scale) || !(scale > 0.f))
     return fail(TK_ERR_INVALID_ARG, "prefill scale must be finite and positive");
   if (desc->batch == 0 || seq == 0) return TK_OK;
-  if ((s = check_cache_ptrs(desc, k_cache, v_cache, nullptr, page_table)) != TK_OK) return s;
+  if ((s = check_cache_ptrs(desc, k_cache, v_cache, k_scale, page_table)) != TK_OK) return s;
   if (!q || !out || !seq_lens || !k_new || !v_new)
     return fail(TK_ERR_INVALID_ARG, "q / out / seq_lens / k_new / v_new is NULL");
   if (!aligned16(q) || !aligned16(out) || !aligned16(k_new) || !aligned16(v_new))
@@ -289,10 +286,11 @@ tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void*
   const cudaStream_t st = static_cast<cudaStream_t>(stream);
   // 1. the chunk's keys and values into the cache at seq_lens[b]
   tk::AppendParams a{};
-  a.k = k_cache; a.v = v_cache; a.k_scale = nullptr; a.page_table = page_table;
+  const bool quant = desc->k_dtype != TK_BF16;
+  a.k = k_cache; a.v = v_cache; a.k_scale = quant ? k_scale : nullptr; a.page_table = page_table;
   a.seq_lens = seq_lens; a.k_new = k_new; a.v_new = v_new; a.err = dev.err;
   a.B = desc->batch; a.Hkv = desc->h_kv; a.R = desc->r; a.DV = desc->d_v; a.T = seq;
-  a.k_fmt = 0;
+  a.k_fmt = key_format(desc->k_dtype);
   a.capacity = desc->capacity;
   a.page_size = desc->page_size;
   a.page_shift = desc->page_size ? log2i(desc->page_size) : 0;
@@ -312,6 +310,8 @@ tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void*
   p.num_sms = dev.num_sms;
   p.seq_lens = seq_lens;
   p.page_table = page_table;
+  p.k_fmt = key_format(desc->k_dtype);
+  p.k_scale = quant ? k_scale : nullptr;
   p.capacity = desc->capacity;
   p.page_size = desc->page_size;
   p.page_shift = a.page_shift;

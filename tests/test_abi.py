@@ -41,7 +41,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert tb.tk_abi_version() == 1
+    assert tb.tk_abi_version() == 2
     assert tb.tk_status_string(tb.TK_OK) == "TK_OK"
     assert tb.tk_status_string(tb.TK_ERR_WORKSPACE) == "TK_ERR_WORKSPACE"
     assert tb.tk_status_string(99) == "TK_ERR_UNKNOWN"
@@ -128,18 +128,19 @@ def test_decode_append_validation(lib):
 def test_prefill_cached_validation(lib):
     P = lib.tk_attn_prefill_cached
     d = _desc()
-    args = (FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, 64, 256, FAKE, tb.TK_BF16, 0.1, 1, None)
     d8 = _desc(k_dtype=tb.TK_I8)
-    assert P(ctypes.byref(d8), *args) == tb.TK_ERR_UNSUPPORTED
-    assert "bf16 keys" in tb.tk_last_error()
-    assert P(ctypes.byref(d), FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, 64, 32, FAKE, tb.TK_BF16,
-             0.1, 1, None) == tb.TK_ERR_INVALID_ARG            # max_seq_len < seq
-    assert P(ctypes.byref(d), None, FAKE, FAKE, None, FAKE, FAKE, FAKE, 64, 256, FAKE, tb.TK_BF16,
-             0.1, 1, None) == tb.TK_ERR_INVALID_ARG            # q is NULL
-    assert P(ctypes.byref(d), FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, 64, 256, FAKE, tb.TK_BF16,
-             -1.0, 1, None) == tb.TK_ERR_INVALID_ARG           # scale <= 0
-    assert P(ctypes.byref(d), None, None, None, None, None, None, None, 0, 0, None, tb.TK_BF16,
-             0.1, 1, None) == tb.TK_OK                          # empty chunk: no-op
+    # int8 keys need their scales
+    assert P(ctypes.byref(d8), FAKE, FAKE, FAKE, None, None, FAKE, FAKE, FAKE, 64, 256, FAKE,
+             tb.TK_BF16, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG
+    assert "k_scale" in tb.tk_last_error()
+    assert P(ctypes.byref(d), FAKE, FAKE, FAKE, None, None, FAKE, FAKE, FAKE, 64, 32, FAKE,
+             tb.TK_BF16, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG            # max_seq_len < seq
+    assert P(ctypes.byref(d), None, FAKE, FAKE, None, None, FAKE, FAKE, FAKE, 64, 256, FAKE,
+             tb.TK_BF16, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG            # q is NULL
+    assert P(ctypes.byref(d), FAKE, FAKE, FAKE, None, None, FAKE, FAKE, FAKE, 64, 256, FAKE,
+             tb.TK_BF16, -1.0, 1, None) == tb.TK_ERR_INVALID_ARG           # scale <= 0
+    assert P(ctypes.byref(d), None, None, None, None, None, None, None, None, 0, 0, None,
+             tb.TK_BF16, 0.1, 1, None) == tb.TK_OK                          # empty chunk: no-op
 
 
 def test_forward_and_backward_validation(lib):

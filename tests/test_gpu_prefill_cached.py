@@ -4,8 +4,11 @@ The chunk's keys and values land in the cache (bit-exact); its queries at
 positions seq_lens[b] + i attend to the cache's first seq_lens[b] + i + 1
 tokens (end-aligned causal) and match the fp64 oracle; paged caches give the
 same bits as a contiguous one, and an empty context gives the plain prefill
-bit for bit.  A 7B-shaped chunk (4096 new tokens after 4096 cached) is
-checked on sampled rows.
+bit for bit.  int8 and int4 key caches (codes and scales written by the
+quantising append) match the oracle on the dequantised keys, again with
+paged = contiguous bit for bit; cache slots past a context may hold NaN.
+A 7B-shaped chunk (4096 new tokens after 4096 cached) is checked on sampled
+rows, with bf16 and with int8 keys.
 """
 
 import math
@@ -16,21 +19,34 @@ import torch
 
 from _helpers import f64, parity, parity_bf16, require_gpu
 from oracle import attention as oa
+from oracle import cache as oc
 from paper_2603_04427_gb300 import binding as tb
 from paper_2603_04427_gb300 import inputs
 
 pytestmark = pytest.mark.gpu
 
 
-def _setup(B, hq, hkv, r, dv, L0, S, seed, ps=0):
+def _setup(B, hq, hkv, r, dv, L0, S, seed, ps=0, kfmt="bf16", garbage=False):
+    """A cache holding each sequence's L0[b] cached tokens (written by tk_kv_append),
+    the chunk's q / k_new / v_new, and every sequence's whole context K / V (bf16,
+    as appended) for the oracle.  garbage: NaN (bf16) / NaN scales everywhere
+    before the context is written, so slots past it hold NaN."""
     cap = (max(L0) + S + 15) // 16 * 16
     n = [l0 + S for l0 in L0]
+    q8, q4 = kfmt == "int8", kfmt == "int4"
     if ps:
         table, n_pages = inputs.paged_layout(n, ps, seed=seed, extra_pages=2)
         cache = tb.ThinKeyCache.allocate(B, hq, hkv, r, dv, page_size=ps, num_pages=n_pages,
-                                         page_table=table)
+                                         page_table=table, k_int8=q8, k_int4=q4)
     else:
-        cache = tb.ThinKeyCache.allocate(B, hq, hkv, r, dv, capacity=cap)
+        cache = tb.ThinKeyCache.allocate(B, hq, hkv, r, dv, capacity=cap, k_int8=q8, k_int4=q4)
+    if garbage:
+        cache.v.fill_(float("nan"))
+        if kfmt == "bf16":
+            cache.k.fill_(float("nan"))
+        else:
+            cache.k.fill_(0x77)
+            cache.k_scale.fill_(float("nan"))
     T = max(L0)
     kc = inputs.normal_bf16((B, hkv, max(T, 1), r), seed, device="cuda")
     vc = inputs.normal_bf16((B, hkv, max(T, 1), dv), seed + 1, device="cuda")
@@ -38,10 +54,12 @@ def _setup(B, hq, hkv, r, dv, L0, S, seed, ps=0):
     for b, l0 in enumerate(L0):   # the cached context of each sequence
         if l0:
             d = cache.desc
+            ks = cache.k_scale
             one = tb.ThinKeyCache(tb.tk_cache_desc(1, hq, hkv, r, dv, d.capacity, d.page_size,
                                                    d.num_pages, d.max_pages_per_seq, d.k_dtype),
                                   cache.k if ps else cache.k[b:b + 1], cache.v if ps else cache.v[b:b + 1],
-                                  None, cache.page_table[b:b + 1].contiguous() if ps else None)
+                                  None if ks is None else (ks if ps else ks[b:b + 1]),
+                                  cache.page_table[b:b + 1].contiguous() if ps else None)
             tb.tk_kv_append(one, kc[b:b + 1, :, :l0].contiguous(), vc[b:b + 1, :, :l0].contiguous(), zero)
     q = inputs.normal_bf16((B, hq, S, r), seed + 2, device="cuda")
     kn = inputs.normal_bf16((B, hkv, S, r), seed + 3, device="cuda")
@@ -53,6 +71,16 @@ def _setup(B, hq, hkv, r, dv, L0, S, seed, ps=0):
         K[b, :, :l0], V[b, :, :l0] = kc[b, :, :l0], vc[b, :, :l0]
         K[b, :, l0:l0 + S], V[b, :, l0:l0 + S] = kn[b], vn[b]
     return cache, q, kn, vn, K, V, max(n)
+
+
+def _keys_for_oracle(K, kfmt):
+    """The keys the kernels see: bf16 as they are, or the oracle's quantiser's
+    codes times scales (per token and kv head), exact in fp64."""
+    if kfmt == "bf16":
+        return f64(K)
+    quant = oc.quantize_int8_per_token if kfmt == "int8" else oc.quantize_int4_per_token
+    codes, sc = quant(K.float().cpu().numpy())
+    return oa.dequantize_keys(codes, sc)
 
 
 def _run(cache, q, kn, vn, L0, max_len, dtype=torch.float32, causal=True):
@@ -127,3 +155,78 @@ def test_7b_chunk_after_4096_cached_sampled():
                                      f64(V[b, h, :p + 1]), 1 / math.sqrt(r))[0])
         got.append(f64(out[b, h, i]))
     parity_bf16(np.stack(got), np.stack(ref), what="7b cached chunk sampled")
+
+
+@pytest.mark.parametrize("kfmt,r,dv", [("int8", 16, 64), ("int8", 32, 128), ("int8", 64, 64),
+                                       ("int8", 128, 128), ("int4", 32, 128), ("int4", 64, 128),
+                                       ("int4", 128, 64)])
+def test_quantised_cached_prefill_matches_oracle(kfmt, r, dv):
+    require_gpu()
+    B, hq, hkv, S = 3, 8, 2, 300
+    L0 = [0, 100, 777]
+    cache, q, kn, vn, K, V, n = _setup(B, hq, hkv, r, dv, L0, S, seed=40 + r + dv, kfmt=kfmt)
+    out = _run(cache, q, kn, vn, L0, n)
+    ref = oa.attention_prefill_cached(f64(q), _keys_for_oracle(K, kfmt), f64(V), L0, 1 / math.sqrt(r))
+    parity(f64(out), ref, what=f"cached prefill {kfmt} keys r={r} dv={dv}")
+    # the chunk's codes and scales are the oracle quantiser's, bit for bit
+    quant = oc.quantize_int8_per_token if kfmt == "int8" else oc.quantize_int4_per_token
+    for b, l0 in enumerate(L0):
+        codes, sc = quant(kn[b].float().cpu().numpy())
+        stored = cache.k[b, :, l0:l0 + S].cpu().numpy()
+        assert np.array_equal(stored, codes if kfmt == "int8" else oc.pack_int4(codes))
+        assert np.array_equal(cache.k_scale[b, :, l0:l0 + S].cpu().numpy().view(np.uint32),
+                              sc.view(np.uint32))
+        assert torch.equal(cache.v[b, :, l0:l0 + S], vn[b])
+
+
+@pytest.mark.parametrize("kfmt", ["int8", "int4"])
+@pytest.mark.parametrize("ps", [16, 64, 256])
+def test_quantised_cached_prefill_paged_equals_contiguous_bitwise(kfmt, ps):
+    require_gpu()
+    B, hq, hkv, r, dv, S = 3, 8, 2, 32, 128, 257
+    L0 = [5, 130, 640]
+    a = _setup(B, hq, hkv, r, dv, L0, S, seed=23, kfmt=kfmt)
+    p = _setup(B, hq, hkv, r, dv, L0, S, seed=23, ps=ps, kfmt=kfmt)
+    out_a = _run(*a[:4], L0, a[6])
+    out_p = _run(*p[:4], L0, p[6])
+    assert torch.equal(out_a, out_p)
+    ref = oa.attention_prefill_cached(f64(a[1]), _keys_for_oracle(a[4], kfmt), f64(a[5]), L0,
+                                      1 / math.sqrt(r))
+    parity(f64(out_p), ref, what=f"paged {kfmt} ps={ps}")
+
+
+@pytest.mark.parametrize("kfmt,ps", [("bf16", 0), ("int8", 0), ("bf16", 64), ("int4", 16)])
+def test_cached_prefill_ignores_garbage_past_the_context(kfmt, ps):
+    """Slots past each context hold NaN (values, bf16 keys, key scales): never weighted."""
+    require_gpu()
+    B, hq, hkv, r, dv, S = 2, 8, 2, 32, 128, 200
+    L0 = [50, 301]
+    cache, q, kn, vn, K, V, n = _setup(B, hq, hkv, r, dv, L0, S, seed=61, ps=ps, kfmt=kfmt,
+                                       garbage=True)
+    out = _run(cache, q, kn, vn, L0, n)
+    assert torch.isfinite(out).all()
+    ref = oa.attention_prefill_cached(f64(q), _keys_for_oracle(K, kfmt), f64(V), L0, 1 / math.sqrt(r))
+    parity(f64(out), ref, what=f"garbage past the context, {kfmt} ps={ps}")
+
+
+def test_7b_chunk_int8_keys_sampled():
+    """The 7B chunk (4096 new after 4096 cached) over an int8 key cache, bf16 out: one row
+    of every other 128-row query tile of every (sequence, head) plane."""
+    require_gpu()
+    B, H, r, dv, S = 2, 32, 32, 128, 4096
+    L0 = [4096, 4096]
+    cache, q, kn, vn, K, V, n = _setup(B, H, H, r, dv, L0, S, seed=1105, kfmt="int8")
+    out = _run(cache, q, kn, vn, L0, n, dtype=torch.bfloat16)
+    Kq = _keys_for_oracle(K, "int8")
+    Vh, qh, oh = V.cpu(), q.cpu(), out.cpu()
+    got, ref = [], []
+    for b in range(B):
+        for h in range(H):
+            rows = [t * 128 + (t * 29 + (b * H + h) * 7) % 128 for t in range(0, S // 128, 2)]
+            vv = f64(Vh[b, h])
+            for i in rows:
+                p = L0[b] + i
+                ref.append(oa.attention_head(f64(qh[b, h, i])[None], Kq[b, h, :p + 1], vv[:p + 1],
+                                             1 / math.sqrt(r))[0])
+                got.append(f64(oh[b, h, i]))
+    parity_bf16(np.stack(got), np.stack(ref), what="7b cached chunk, int8 keys")
