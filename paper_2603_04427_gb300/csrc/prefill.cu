@@ -99,11 +99,11 @@ struct PCfg {
   static constexpr int OFF_K = 2 * QBA;
   static constexpr int KBA = (KB + 1023) / 1024 * 1024;
   static constexpr int STAGE = KBA + VB;
-  static constexpr int NST = (2 * QBA + 3 * (STAGE + SCB) + STGB + 2048 <= 200 * 1024) ? 3 : 2;
-  // one staging area serves every stage (the TMA warp widens a tile's codes
-  // before it loads the next tile's); the scales keep one slot per stage
+  static constexpr int NST = (2 * QBA + 3 * (STAGE + SCB) + 2 * STGB + 2048 <= 200 * 1024) ? 3 : 2;
+  // two staging slots serve the whole ring (the TMA warp widens tile j's codes
+  // at most one tile behind their load); the scales keep one slot per stage
   static constexpr int OFF_STG = OFF_K + NST * STAGE;
-  static constexpr int OFF_SC = OFF_STG + STGB;
+  static constexpr int OFF_SC = OFF_STG + 2 * STGB;
   static constexpr int OFF_BAR = OFF_SC + NST * SCB;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;      // + slack to align the base to 1 KB
   static_assert(SMEM <= 227 * 1024, "shared memory");
@@ -259,11 +259,20 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
           tma_load_3d(smem + C::OFF_Q + x * C::QBA + i * C::QK_BOXB, &maps.q, i * C::QK_BOX,
                       (qa + x) * kBM, bh, q_full);
     }
-    for (int j = 0; j < n_kv; ++j) {
+    // A tile is "relayed" when this warp must finish it before the MMA warp may
+    // read it: every tile of a quantised cache (codes widened to bf16) and, in
+    // cached mode, the tile holding the context's end (value rows past it zeroed:
+    // the cache may hold anything there, and 0 * NaN would spread).  Other tiles
+    // go straight from the TMA to k_full.
+    auto relayed = [&](int j) {
+      return relay && (KF != kKeyBF16 || kv_len - j * kBN < kBN);
+    };
+    // issue(j): wait for the stage, then the TMA loads of tile j
+    auto issue = [&](int j) -> bool {
       const int st = j % NST;
       int okw = 1;
       if (j >= NST && lane == 0) okw = mbar_wait(&kv_empty[st], ((j / NST) - 1) & 1, p.err);
-      if (!__shfl_sync(0xffffffffu, okw, 0)) break;
+      if (!__shfl_sync(0xffffffffu, okw, 0)) return false;
       // lane s < nsub finds the plane and first row of sub-box s
       int plane = kv_plane, row = j * kBN;
       if (p.page_size != 0) {
@@ -285,24 +294,19 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
         planes[s2] = __shfl_sync(0xffffffffu, plane, s2);
         rows[s2] = __shfl_sync(0xffffffffu, row, s2);
       }
-      unsigned char* sk = smem + C::OFF_K + st * C::STAGE;
-      unsigned char* sv = sk + C::KBA;
       if (lane == 0) {
-        if (!relay) {
-          mbar_arrive_expect_tx(&k_full[st], C::KB);
+        unsigned char* sk = smem + C::OFF_K + st * C::STAGE;
+        unsigned char* sv = sk + C::KBA;
+        if constexpr (KF == kKeyBF16) {
+          uint64_t* kb = relayed(j) ? &c_full[st] : &k_full[st];
+          mbar_arrive_expect_tx(kb, C::KB);
           for (int s2 = 0; s2 < nsub; ++s2)
             for (int i = 0; i < C::QK_NBOX; ++i)
               tma_load_3d(sk + i * C::QK_BOXB + s2 * bps * C::QK_SW, &maps.k, i * C::QK_BOX,
-                          rows[s2], planes[s2], &k_full[st]);
-        } else if constexpr (KF == kKeyBF16) {
-          mbar_arrive_expect_tx(&c_full[st], C::KB);
-          for (int s2 = 0; s2 < nsub; ++s2)
-            for (int i = 0; i < C::QK_NBOX; ++i)
-              tma_load_3d(sk + i * C::QK_BOXB + s2 * bps * C::QK_SW, &maps.k, i * C::QK_BOX,
-                          rows[s2], planes[s2], &c_full[st]);
+                          rows[s2], planes[s2], kb);
         } else {
-          // raw codes into the staging area, the tile's key scales after them
-          unsigned char* stg = smem + C::OFF_STG;
+          // raw codes into staging slot j % 2, the tile's key scales into the stage's slot
+          unsigned char* stg = smem + C::OFF_STG + (j & 1) * C::STGB;
           float* sc = reinterpret_cast<float*>(smem + C::OFF_SC + st * C::SCB);
           const int kv0 = j * kBN;
           uint32_t sc_bytes = 0;
@@ -332,47 +336,62 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
             tma_load_3d(sv + i * C::V_BOXB + s2 * bps * 128, &maps.v, i * 64, rows[s2], planes[s2],
                         &v_full[st]);
       }
-      if (relay) {
-        // Cached mode: the warp finishes the K tile before the MMA warp may read
-        // it -- quantised codes are widened to bf16 in the tile's swizzled layout,
-        // and on the tile that holds the context's end the value rows past it are
-        // zeroed (the cache may hold anything there, and 0 * NaN would spread).
-        const uint32_t ph = (j / NST) & 1;
-        bool okc = mbar_wait(&c_full[st], ph, p.err);
-        const int kv0 = j * kBN, n_valid = kv_len - kv0;
-        if (n_valid < kBN) okc = mbar_wait(&v_full[st], ph, p.err) && okc;
-        if (!__all_sync(0xffffffffu, okc)) break;
-        if constexpr (KF != kKeyBF16) {
-          const unsigned char* stg = smem + C::OFF_STG;
-          constexpr int PPR = R / 8;  // 16-byte bf16 pieces per key row
+      return true;
+    };
+    // finish(j) of a relayed tile: widen its codes, zero value rows past the
+    // context, then publish the K tile on k_full
+    auto finish = [&](int j) -> bool {
+      const int st = j % NST;
+      unsigned char* sk = smem + C::OFF_K + st * C::STAGE;
+      unsigned char* sv = sk + C::KBA;
+      // quantised caches use c_full on every tile; a bf16 cache only on its last
+      const uint32_t phc = KF != kKeyBF16 ? (j / NST) & 1 : 0;
+      bool okc = mbar_wait(&c_full[st], phc, p.err);
+      const int n_valid = kv_len - j * kBN;
+      if (n_valid < kBN) okc = mbar_wait(&v_full[st], (j / NST) & 1, p.err) && okc;
+      if (!__all_sync(0xffffffffu, okc)) return false;
+      if constexpr (KF != kKeyBF16) {
+        const unsigned char* stg = smem + C::OFF_STG + (j & 1) * C::STGB;
+        constexpr int PPR = R / 8;  // 16-byte bf16 pieces per key row
 #pragma unroll 4
-          for (int c = lane; c < kBN * PPR; c += 32) {
-            const int row = c / PPR, e0 = (c % PPR) * 8;
-            uint2 lo, hi;
-            if constexpr (KF == kKeyInt8) {
-              const uint2 w = *reinterpret_cast<const uint2*>(stg + row * C::CODE_ROWB + e0);
-              lo = int8x4_to_bf16(w.x);
-              hi = int8x4_to_bf16(w.y);
-            } else {
-              const uint32_t w = *reinterpret_cast<const uint32_t*>(stg + row * C::CODE_ROWB + e0 / 2);
-              lo = int4x4_to_bf16(w & 0xffffu);
-              hi = int4x4_to_bf16(w >> 16);
-            }
-            *reinterpret_cast<uint4*>(sk + k_piece_offset<C>(row, e0)) = make_uint4(lo.x, lo.y, hi.x, hi.y);
+        for (int c = lane; c < kBN * PPR; c += 32) {
+          const int row = c / PPR, e0 = (c % PPR) * 8;
+          uint2 lo, hi;
+          if constexpr (KF == kKeyInt8) {
+            const uint2 w = *reinterpret_cast<const uint2*>(stg + row * C::CODE_ROWB + e0);
+            lo = int8x4_to_bf16(w.x);
+            hi = int8x4_to_bf16(w.y);
+          } else {
+            const uint32_t w = *reinterpret_cast<const uint32_t*>(stg + row * C::CODE_ROWB + e0 / 2);
+            lo = int4x4_to_bf16(w & 0xffffu);
+            hi = int4x4_to_bf16(w >> 16);
           }
+          *reinterpret_cast<uint4*>(sk + k_piece_offset<C>(row, e0)) = make_uint4(lo.x, lo.y, hi.x, hi.y);
         }
-        if (n_valid < kBN) {
-          const int first = max(n_valid, 0);
-          for (int c = lane; c < (kBN - first) * 8 * C::V_NBOX; c += 32) {
-            const int box = c / ((kBN - first) * 8), rem2 = c % ((kBN - first) * 8);
-            *reinterpret_cast<uint4*>(sv + box * C::V_BOXB + (first + rem2 / 8) * 128 + (rem2 % 8) * 16) =
-                make_uint4(0u, 0u, 0u, 0u);
-          }
-        }
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&k_full[st]);
       }
+      if (n_valid < kBN) {
+        const int first = max(n_valid, 0);
+        const int per_box = (kBN - first) * 8;   // 16-byte pieces per value box
+        for (int c = lane; c < per_box * C::V_NBOX; c += 32) {
+          const int box = c / per_box, rem2 = c % per_box;
+          *reinterpret_cast<uint4*>(sv + box * C::V_BOXB + (first + rem2 / 8) * 128 + (rem2 % 8) * 16) =
+              make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&k_full[st]);
+      return true;
+    };
+    // Quantised tiles are finished one tile behind their loads, so the next
+    // tile's TMA is in flight while this one is widened.  That needs a third
+    // ring stage: with two, loading tile j+1 waits for the release of tile
+    // j-1, which waits for the scores of tile j, i.e. for finish(j).
+    constexpr int LAG = (KF != kKeyBF16 && NST >= 3) ? 1 : 0;
+    for (int j = 0; j < n_kv + LAG; ++j) {
+      if (j < n_kv && !issue(j)) break;
+      const int jf = j - LAG;
+      if (jf >= 0 && relayed(jf) && !finish(jf)) break;
     }
   } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer
@@ -467,10 +486,14 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
           const float4 f = sc4[i];
-          v[4 * i] = __float_as_uint(__uint_as_float(v[4 * i]) * f.x);
-          v[4 * i + 1] = __float_as_uint(__uint_as_float(v[4 * i + 1]) * f.y);
-          v[4 * i + 2] = __float_as_uint(__uint_as_float(v[4 * i + 2]) * f.z);
-          v[4 * i + 3] = __float_as_uint(__uint_as_float(v[4 * i + 3]) * f.w);
+          const float2 a = fmul2(make_float2(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1])),
+                                 make_float2(f.x, f.y));
+          const float2 c = fmul2(make_float2(__uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3])),
+                                 make_float2(f.z, f.w));
+          v[4 * i] = __float_as_uint(a.x);
+          v[4 * i + 1] = __float_as_uint(a.y);
+          v[4 * i + 2] = __float_as_uint(c.x);
+          v[4 * i + 3] = __float_as_uint(c.y);
         }
       }
       if (masked) {
