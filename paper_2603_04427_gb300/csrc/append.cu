@@ -6,8 +6,11 @@
 // variant is the composition with key quantisation of Section 6 (the scheme
 // is in kv_row.cuh).
 //
-// One warp per (b, g, t): 16-byte vector loads and stores for bf16 rows; for
-// int8 keys a warp max-reduction gives amax.
+// One warp per run of kRows consecutive tokens of one (b, g): every 16-byte
+// piece of the run's bf16 rows is loaded before any is stored, so a warp has
+// kRows rows in flight (one row per warp leaves the copy far below the HBM
+// rate: too few bytes in flight per SM).  Quantised keys are then written row
+// by row (a warp max-reduction gives each row's amax).
 #include "common.cuh"
 #include "kernels.h"
 #include "kv_row.cuh"
@@ -16,49 +19,91 @@ namespace tk {
 namespace {
 
 constexpr int kWarps = 4;
+constexpr int kRows = 8;   // tokens per warp
 
 template <int R, int DV, int KF>
 __global__ void __launch_bounds__(kWarps * 32) append_kernel(const AppendParams p) {
   const int lane = threadIdx.x & 31;
   const long wg = static_cast<long>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
-  const long total = static_cast<long>(p.B) * p.Hkv * p.T;
+  const int n_runs = (p.T + kRows - 1) / kRows;
+  const long total = static_cast<long>(p.B) * p.Hkv * n_runs;
   if (wg >= total) return;
   pdl_wait();
   pdl_trigger();
-  const int t = static_cast<int>(wg % p.T);
-  const int g = static_cast<int>((wg / p.T) % p.Hkv);
-  const int b = static_cast<int>(wg / (static_cast<long>(p.T) * p.Hkv));
-  const int pos = p.seq_lens[b] + t;
+  const int t0 = static_cast<int>(wg % n_runs) * kRows;
+  const int g = static_cast<int>((wg / n_runs) % p.Hkv);
+  const int b = static_cast<int>(wg / (static_cast<long>(n_runs) * p.Hkv));
+  const int pos0 = p.seq_lens[b] + t0;
 
-  size_t row;  // destination row in the cache / pool
-  if (p.page_size == 0) {
-    if (pos < 0 || pos >= p.capacity) {
-      if (lane == 0) record_error(p.err, TK_DEVERR_INDEX);
-      return;
+  // destination row of token t0 + i in the cache / pool, or -1 (past the run's
+  // end, or out of range: recorded)
+  auto dst_row = [&](int i) -> long long {
+    const int pos = pos0 + i;
+    if (t0 + i >= p.T) return -1;
+    if (p.page_size == 0) {
+      if (pos < 0 || pos >= p.capacity) {
+        record_error(p.err, TK_DEVERR_INDEX);
+        return -1;
+      }
+      return (static_cast<long long>(b) * p.Hkv + g) * p.capacity + pos;
     }
-    row = (static_cast<size_t>(b) * p.Hkv + g) * p.capacity + pos;
-  } else {
     const int pidx = pos >> p.page_shift;
     if (pos < 0 || pidx >= p.max_pages) {
-      if (lane == 0) record_error(p.err, TK_DEVERR_INDEX);
-      return;
+      record_error(p.err, TK_DEVERR_INDEX);
+      return -1;
     }
     const int page = p.page_table[static_cast<size_t>(b) * p.max_pages + pidx];
     if (page < 0 || page >= p.num_pages) {
-      if (lane == 0) record_error(p.err, TK_DEVERR_INDEX);
-      return;
+      record_error(p.err, TK_DEVERR_INDEX);
+      return -1;
     }
-    row = (static_cast<size_t>(page) * p.Hkv + g) * p.page_size + (pos & (p.page_size - 1));
+    return (static_cast<long long>(page) * p.Hkv + g) * p.page_size + (pos & (p.page_size - 1));
+  };
+  const size_t src0 = (static_cast<size_t>(b) * p.Hkv + g) * p.T + t0;
+  const uint4* vs = static_cast<const uint4*>(p.v_new) + src0 * (2 * DV / 16);
+  const uint4* ks = static_cast<const uint4*>(p.k_new) + src0 * (2 * R / 16);
+  uint4* vd = static_cast<uint4*>(p.v);
+  uint4* kd = static_cast<uint4*>(p.k);
+  // values (and bf16 keys): piece c of the run = row c / N, piece c % N of that row
+  constexpr int NV = 2 * DV / 16, NK = 2 * R / 16;
+  constexpr int PV = (kRows * NV + 31) / 32, PK = (kRows * NK + 31) / 32;
+  uint4 vr[PV], kr[PK];
+  long long vdst[PV], kdst[PK];
+#pragma unroll
+  for (int i = 0; i < PV; ++i) {
+    const int c = lane + 32 * i;
+    vdst[i] = c < kRows * NV ? dst_row(c / NV) : -1;
+    if (vdst[i] >= 0) vr[i] = vs[c];
   }
-  const size_t src = (static_cast<size_t>(b) * p.Hkv + g) * p.T + t;
-  write_kv_row<R, DV, KF>(p.k, p.v, p.k_scale, row,
-                           static_cast<const unsigned char*>(p.k_new) + src * 2 * R,
-                           static_cast<const unsigned char*>(p.v_new) + src * 2 * DV, lane);
+  if constexpr (KF == 0) {
+#pragma unroll
+    for (int i = 0; i < PK; ++i) {
+      const int c = lane + 32 * i;
+      kdst[i] = c < kRows * NK ? dst_row(c / NK) : -1;
+      if (kdst[i] >= 0) kr[i] = ks[c];
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < PV; ++i)
+    if (vdst[i] >= 0) vd[vdst[i] * NV + (lane + 32 * i) % NV] = vr[i];
+  if constexpr (KF == 0) {
+#pragma unroll
+    for (int i = 0; i < PK; ++i)
+      if (kdst[i] >= 0) kd[kdst[i] * NK + (lane + 32 * i) % NK] = kr[i];
+  } else {
+#pragma unroll 1
+    for (int i = 0; i < kRows; ++i) {
+      const long long d = dst_row(i);
+      if (d >= 0)
+        write_k_row<R, KF>(p.k, p.k_scale, static_cast<size_t>(d),
+                           static_cast<const unsigned char*>(p.k_new) + (src0 + i) * 2 * R, lane);
+    }
+  }
 }
 
 template <int R, int DV, int KF>
 cudaError_t launch_t(const AppendParams& p, cudaStream_t s) {
-  const long warps = static_cast<long>(p.B) * p.Hkv * p.T;
+  const long warps = static_cast<long>(p.B) * p.Hkv * ((p.T + kRows - 1) / kRows);
   const long blocks = (warps + kWarps - 1) / kWarps;
   if (blocks > 0x7fffffffL) return cudaErrorInvalidConfiguration;
   return launch_pdl(append_kernel<R, DV, KF>, dim3(static_cast<unsigned>(blocks)),

@@ -16,18 +16,19 @@
 
 namespace tk {
 
-// KF: key format, 0 bf16, 1 int8, 2 int4 (R >= 32).
-template <int R, int DV, int KF>
-__device__ __forceinline__ void write_kv_row(void* k_cache, void* v_cache, float* k_scale,
-                                             size_t row, const void* k_src, const void* v_src,
-                                             int lane) {
-  // values: d_v bf16 = 2 * DV bytes, 16 bytes per lane
-  {
-    constexpr int NV = 2 * DV / 16;
-    const uint4* s = static_cast<const uint4*>(v_src);
-    uint4* d = reinterpret_cast<uint4*>(static_cast<unsigned char*>(v_cache) + row * 2 * DV);
-    if (lane < NV) d[lane] = s[lane];
-  }
+// The value row: d_v bf16 = 2 * DV bytes, 16 bytes per lane.
+template <int DV>
+__device__ __forceinline__ void write_v_row(void* v_cache, size_t row, const void* v_src, int lane) {
+  constexpr int NV = 2 * DV / 16;
+  const uint4* s = static_cast<const uint4*>(v_src);
+  uint4* d = reinterpret_cast<uint4*>(static_cast<unsigned char*>(v_cache) + row * 2 * DV);
+  if (lane < NV) d[lane] = s[lane];
+}
+
+// The key row.  KF: key format, 0 bf16, 1 int8, 2 int4 (R >= 32).
+template <int R, int KF>
+__device__ __forceinline__ void write_k_row(void* k_cache, float* k_scale, size_t row,
+                                            const void* k_src, int lane) {
   if constexpr (KF == 0) {
     constexpr int NK = 2 * R / 16;
     const uint4* s = static_cast<const uint4*>(k_src);
@@ -78,6 +79,15 @@ __device__ __forceinline__ void write_kv_row(void* k_cache, void* v_cache, float
     }
     if (lane == 0) k_scale[row] = scale;
   }
+}
+
+// The whole cache row of one token: value, then key.
+template <int R, int DV, int KF>
+__device__ __forceinline__ void write_kv_row(void* k_cache, void* v_cache, float* k_scale,
+                                             size_t row, const void* k_src, const void* v_src,
+                                             int lane) {
+  write_v_row<DV>(v_cache, row, v_src, lane);
+  write_k_row<R, KF>(k_cache, k_scale, row, k_src, lane);
 }
 
 }  // namespace tk

@@ -31,6 +31,7 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "tc05.cuh"
+#include "widen.cuh"
 
 namespace tk {
 namespace {
@@ -120,32 +121,6 @@ __device__ __forceinline__ uint32_t k_piece_offset(int row, int e0) {
   const uint32_t o = static_cast<uint32_t>(row * C::QK_SW + (e0 % C::QK_BOX) * 2);
   constexpr uint32_t mask = static_cast<uint32_t>(C::QK_SW / 16 - 1) << 4;
   return static_cast<uint32_t>((e0 / C::QK_BOX) * C::QK_BOXB) + (o ^ ((o >> 3) & mask));
-}
-
-// Four int8 codes (one per byte) -> two words of two bf16 each (element 4i in the
-// low half of the first word); exact: |code| <= 127 is a bf16 value.
-__device__ __forceinline__ uint2 int8x4_to_bf16(uint32_t w) {
-  float f[4];
-#pragma unroll
-  for (int i = 0; i < 4; ++i)
-    f[i] = static_cast<float>(static_cast<int>(static_cast<int8_t>((w >> (8 * i)) & 0xffu)));
-  __nv_bfloat162 a = __floats2bfloat162_rn(f[0], f[1]), b = __floats2bfloat162_rn(f[2], f[3]);
-  return make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&b));
-}
-
-// Two bytes of packed int4 codes (element 2j in the low nibble of byte j, 2j+1 in
-// the high nibble, 4-bit two's complement) -> two words of two bf16 each; exact.
-__device__ __forceinline__ uint2 int4x4_to_bf16(uint32_t two_bytes) {
-  int c[4];
-#pragma unroll
-  for (int i = 0; i < 2; ++i) {
-    const int b = static_cast<int>((two_bytes >> (8 * i)) & 0xffu);
-    c[2 * i] = static_cast<int>(static_cast<int8_t>(b << 4)) >> 4;
-    c[2 * i + 1] = static_cast<int>(static_cast<int8_t>(b)) >> 4;
-  }
-  __nv_bfloat162 a = __floats2bfloat162_rn(static_cast<float>(c[0]), static_cast<float>(c[1]));
-  __nv_bfloat162 d = __floats2bfloat162_rn(static_cast<float>(c[2]), static_cast<float>(c[3]));
-  return make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&d));
 }
 
 struct Maps {
@@ -356,17 +331,18 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
 #pragma unroll 4
         for (int c = lane; c < kBN * PPR; c += 32) {
           const int row = c / PPR, e0 = (c % PPR) * 8;
-          uint2 lo, hi;
+          // exact widening by integer moves (no int-to-float conversions, which
+          // would share the ex2 unit with the softmax warps)
+          uint4 o;
           if constexpr (KF == kKeyInt8) {
             const uint2 w = *reinterpret_cast<const uint2*>(stg + row * C::CODE_ROWB + e0);
-            lo = int8x4_to_bf16(w.x);
-            hi = int8x4_to_bf16(w.y);
+            i8x4_to_bf16(w.x, o.x, o.y);
+            i8x4_to_bf16(w.y, o.z, o.w);
           } else {
             const uint32_t w = *reinterpret_cast<const uint32_t*>(stg + row * C::CODE_ROWB + e0 / 2);
-            lo = int4x4_to_bf16(w & 0xffffu);
-            hi = int4x4_to_bf16(w >> 16);
+            i4x8_to_bf16(w, o.x, o.y, o.z, o.w);
           }
-          *reinterpret_cast<uint4*>(sk + k_piece_offset<C>(row, e0)) = make_uint4(lo.x, lo.y, hi.x, hi.y);
+          *reinterpret_cast<uint4*>(sk + k_piece_offset<C>(row, e0)) = o;
         }
       }
       if (n_valid < kBN) {
