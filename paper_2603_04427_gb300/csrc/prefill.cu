@@ -19,6 +19,8 @@
 //     read S from TMEM, apply the causal / length mask, keep the running max m
 //     and sum l (log2 domain), write P = exp2(S * scale*log2e - m) as bf16 into
 //     the first 64 TMEM columns of S, and at the end write O / l.
+//   warps 10-11 (int8 / int4 key caches only): widen each K tile's codes to
+//     bf16 in the swizzled operand layout, half a tile each.
 // The running max is updated lazily: O and l are rescaled only when a tile's
 // maximum exceeds the max in use by more than 8 (a factor 256), so the
 // weights stay <= 256 and the result is unchanged (O / l uses one consistent
@@ -39,6 +41,9 @@ namespace {
 constexpr int kBM = 128;          // query rows per tile
 constexpr int kBN = 128;          // keys per kv tile
 constexpr int kThreads = 320;     // 2 x 4 softmax warps, 1 TMA warp, 1 MMA warp
+// quantised-key caches add two warps that widen the key codes of each tile
+template <int KF>
+constexpr int threads_for() { return KF == 0 ? kThreads : kThreads + 64; }
 constexpr int kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 // P of a tile is published in kParts key ranges, so the P V products of one
@@ -101,10 +106,12 @@ struct PCfg {
   static constexpr int KBA = (KB + 1023) / 1024 * 1024;
   static constexpr int STAGE = KBA + VB;
   static constexpr int NST = (2 * QBA + 3 * (STAGE + SCB) + 2 * STGB + 2048 <= 200 * 1024) ? 3 : 2;
-  // two staging slots serve the whole ring (the TMA warp widens tile j's codes
-  // at most one tile behind their load); the scales keep one slot per stage
+  // raw codes wait in a staging slot until the widening warps have widened
+  // them: one slot per stage where shared memory allows, else two slots that
+  // the TMA warp reuses once they are free; the scales keep one slot per stage
+  static constexpr int NSTG = (2 * QBA + NST * (STAGE + SCB + STGB) + 2048 <= 200 * 1024) ? NST : 2;
   static constexpr int OFF_STG = OFF_K + NST * STAGE;
-  static constexpr int OFF_SC = OFF_STG + 2 * STGB;
+  static constexpr int OFF_SC = OFF_STG + NSTG * STGB;
   static constexpr int OFF_BAR = OFF_SC + NST * SCB;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;      // + slack to align the base to 1 KB
   static_assert(SMEM <= 227 * 1024, "shared memory");
@@ -139,7 +146,7 @@ struct Maps {
 //   warp 8: TMA producer (Q tiles once, K/V tiles into an NST-stage ring)
 //   warp 9: MMA issuer
 template <int R, int DV, int KF>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(threads_for<KF>(), 1)
 prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   using C = PCfg<R, DV, KF>;
   constexpr int NST = C::NST;
@@ -155,7 +162,8 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   uint64_t* p_full = s_full + 2;                // [tile][part]: P of one key range
   uint64_t* o_full = p_full + 2 * kParts;       // [2]
   uint64_t* c_full = o_full + 2;                // [NST] cached mode: raw K tile (+ scales) landed
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(c_full + NST);
+  uint64_t* stg_free = c_full + NST;            // [NSTG] quantised keys: staging slot widened
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(stg_free + C::NSTG);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int n_qt = (p.S + kBM - 1) / kBM;
@@ -195,11 +203,13 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   if (tid == 0) {
     mbar_init(q_full, 1);
     for (int s = 0; s < NST; ++s) {
-      mbar_init(&k_full[s], 1);
+      // quantised keys: both widening warps arrive on k_full; otherwise the TMA warp
+      mbar_init(&k_full[s], KF == kKeyBF16 ? 1 : 2);
       mbar_init(&v_full[s], 1);
       mbar_init(&kv_empty[s], 1);
       mbar_init(&c_full[s], 1);
     }
+    for (int s = 0; s < C::NSTG; ++s) mbar_init(&stg_free[s], 2);
     for (int x = 0; x < 2; ++x) {
       mbar_init(&s_full[x], 1);
       for (int h = 0; h < kParts; ++h) mbar_init(&p_full[kParts * x + h], 128);
@@ -215,6 +225,67 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
+  // A tile is "relayed" when it must be finished in shared memory before the MMA
+  // warp may read it: every tile of a quantised cache (codes widened to bf16,
+  // by the two widening warps) and, in cached mode, the tile holding the
+  // context's end (value rows past it zeroed by the TMA warp: the cache may hold
+  // anything there, and 0 * NaN would spread).  Other tiles go straight from the
+  // TMA to k_full.
+  const bool relay = p.seq_lens != nullptr;
+  auto relayed = [&](int j) {
+    return relay && (KF != kKeyBF16 || kv_len - j * kBN < kBN);
+  };
+  // finish(j, part, nparts) of a relayed tile, by warp `part` of the nparts
+  // warps that share it: widen its share of the codes, zero its share of the
+  // value rows past the context, then publish on k_full (nparts arrivals)
+  auto finish = [&](int j, int part, int nparts) -> bool {
+    const int st = j % NST;
+    unsigned char* sk = smem + C::OFF_K + st * C::STAGE;
+    unsigned char* sv = sk + C::KBA;
+    // quantised caches use c_full on every tile; a bf16 cache only on its last
+    const uint32_t phc = KF != kKeyBF16 ? (j / NST) & 1 : 0;
+    bool okc = mbar_wait(&c_full[st], phc, p.err);
+    const int n_valid = kv_len - j * kBN;
+    if (n_valid < kBN) okc = mbar_wait(&v_full[st], (j / NST) & 1, p.err) && okc;
+    if (!__all_sync(0xffffffffu, okc)) return false;
+    if constexpr (KF != kKeyBF16) {
+      const unsigned char* stg = smem + C::OFF_STG + (j % C::NSTG) * C::STGB;
+      constexpr int PPR = R / 8;  // 16-byte bf16 pieces per key row
+#pragma unroll 4
+      for (int c = part * 32 + lane; c < kBN * PPR; c += 32 * nparts) {
+        const int row = c / PPR, e0 = (c % PPR) * 8;
+        // exact widening by integer moves (no int-to-float conversions, which
+        // would share the ex2 unit with the softmax warps)
+        uint4 o;
+        if constexpr (KF == kKeyInt8) {
+          const uint2 w = *reinterpret_cast<const uint2*>(stg + row * C::CODE_ROWB + e0);
+          i8x4_to_bf16(w.x, o.x, o.y);
+          i8x4_to_bf16(w.y, o.z, o.w);
+        } else {
+          const uint32_t w = *reinterpret_cast<const uint32_t*>(stg + row * C::CODE_ROWB + e0 / 2);
+          i4x8_to_bf16(w, o.x, o.y, o.z, o.w);
+        }
+        *reinterpret_cast<uint4*>(sk + k_piece_offset<C>(row, e0)) = o;
+      }
+    }
+    if (n_valid < kBN) {
+      const int first = max(n_valid, 0);
+      const int per_box = (kBN - first) * 8;   // 16-byte pieces per value box
+      for (int c = part * 32 + lane; c < per_box * C::V_NBOX; c += 32 * nparts) {
+        const int box = c / per_box, rem2 = c % per_box;
+        *reinterpret_cast<uint4*>(sv + box * C::V_BOXB + (first + rem2 / 8) * 128 + (rem2 % 8) * 16) =
+            make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    __syncwarp();
+    if (lane == 0) {
+      mbar_arrive(&k_full[st]);
+      if constexpr (KF != kKeyBF16) mbar_arrive(&stg_free[j % C::NSTG]);  // staging slot read
+    }
+    return true;
+  };
+
   if (warp == 8) {
     // ------------------------------------------------------------------ TMA producer
     // K/V maps are [planes][rows][width]: plane b*Hkv + g with rows = S (plain) or
@@ -223,7 +294,6 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
     const int g = h / (p.Hq / p.Hkv);
     const int bps = (p.page_size == 0 || p.page_size >= kBN) ? kBN : p.page_size;
     const int nsub = kBN / bps;
-    const bool relay = p.seq_lens != nullptr;   // cached mode: K tiles pass through this warp
     if (lane == 0) {
       prefetch_map(&maps.q);
       prefetch_map(&maps.k);
@@ -234,19 +304,14 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
           tma_load_3d(smem + C::OFF_Q + x * C::QBA + i * C::QK_BOXB, &maps.q, i * C::QK_BOX,
                       (qa + x) * kBM, bh, q_full);
     }
-    // A tile is "relayed" when this warp must finish it before the MMA warp may
-    // read it: every tile of a quantised cache (codes widened to bf16) and, in
-    // cached mode, the tile holding the context's end (value rows past it zeroed:
-    // the cache may hold anything there, and 0 * NaN would spread).  Other tiles
-    // go straight from the TMA to k_full.
-    auto relayed = [&](int j) {
-      return relay && (KF != kKeyBF16 || kv_len - j * kBN < kBN);
-    };
     // issue(j): wait for the stage, then the TMA loads of tile j
     auto issue = [&](int j) -> bool {
       const int st = j % NST;
       int okw = 1;
       if (j >= NST && lane == 0) okw = mbar_wait(&kv_empty[st], ((j / NST) - 1) & 1, p.err);
+      // quantised keys: staging slot j % NSTG must have been widened (tile j - NSTG)
+      if (KF != kKeyBF16 && j >= C::NSTG && lane == 0 && okw)
+        okw = mbar_wait(&stg_free[j % C::NSTG], ((j / C::NSTG) - 1) & 1, p.err);
       if (!__shfl_sync(0xffffffffu, okw, 0)) return false;
       // lane s < nsub finds the plane and first row of sub-box s
       int plane = kv_plane, row = j * kBN;
@@ -280,8 +345,9 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
               tma_load_3d(sk + i * C::QK_BOXB + s2 * bps * C::QK_SW, &maps.k, i * C::QK_BOX,
                           rows[s2], planes[s2], kb);
         } else {
-          // raw codes into staging slot j % 2, the tile's key scales into the stage's slot
-          unsigned char* stg = smem + C::OFF_STG + (j & 1) * C::STGB;
+          // raw codes into staging slot j % NSTG (emptied by the widening warps,
+          // waited for above), the tile's key scales into the stage's slot
+          unsigned char* stg = smem + C::OFF_STG + (j % C::NSTG) * C::STGB;
           float* sc = reinterpret_cast<float*>(smem + C::OFF_SC + st * C::SCB);
           const int kv0 = j * kBN;
           uint32_t sc_bytes = 0;
@@ -313,62 +379,20 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       }
       return true;
     };
-    // finish(j) of a relayed tile: widen its codes, zero value rows past the
-    // context, then publish the K tile on k_full
-    auto finish = [&](int j) -> bool {
-      const int st = j % NST;
-      unsigned char* sk = smem + C::OFF_K + st * C::STAGE;
-      unsigned char* sv = sk + C::KBA;
-      // quantised caches use c_full on every tile; a bf16 cache only on its last
-      const uint32_t phc = KF != kKeyBF16 ? (j / NST) & 1 : 0;
-      bool okc = mbar_wait(&c_full[st], phc, p.err);
-      const int n_valid = kv_len - j * kBN;
-      if (n_valid < kBN) okc = mbar_wait(&v_full[st], (j / NST) & 1, p.err) && okc;
-      if (!__all_sync(0xffffffffu, okc)) return false;
-      if constexpr (KF != kKeyBF16) {
-        const unsigned char* stg = smem + C::OFF_STG + (j & 1) * C::STGB;
-        constexpr int PPR = R / 8;  // 16-byte bf16 pieces per key row
-#pragma unroll 4
-        for (int c = lane; c < kBN * PPR; c += 32) {
-          const int row = c / PPR, e0 = (c % PPR) * 8;
-          // exact widening by integer moves (no int-to-float conversions, which
-          // would share the ex2 unit with the softmax warps)
-          uint4 o;
-          if constexpr (KF == kKeyInt8) {
-            const uint2 w = *reinterpret_cast<const uint2*>(stg + row * C::CODE_ROWB + e0);
-            i8x4_to_bf16(w.x, o.x, o.y);
-            i8x4_to_bf16(w.y, o.z, o.w);
-          } else {
-            const uint32_t w = *reinterpret_cast<const uint32_t*>(stg + row * C::CODE_ROWB + e0 / 2);
-            i4x8_to_bf16(w, o.x, o.y, o.z, o.w);
-          }
-          *reinterpret_cast<uint4*>(sk + k_piece_offset<C>(row, e0)) = o;
-        }
+    if constexpr (KF == kKeyBF16) {
+      for (int j = 0; j < n_kv; ++j) {
+        if (!issue(j)) break;
+        if (relayed(j) && !finish(j, 0, 1)) break;
       }
-      if (n_valid < kBN) {
-        const int first = max(n_valid, 0);
-        const int per_box = (kBN - first) * 8;   // 16-byte pieces per value box
-        for (int c = lane; c < per_box * C::V_NBOX; c += 32) {
-          const int box = c / per_box, rem2 = c % per_box;
-          *reinterpret_cast<uint4*>(sv + box * C::V_BOXB + (first + rem2 / 8) * 128 + (rem2 % 8) * 16) =
-              make_uint4(0u, 0u, 0u, 0u);
-        }
-      }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&k_full[st]);
-      return true;
-    };
-    // Quantised tiles are finished one tile behind their loads, so the next
-    // tile's TMA is in flight while this one is widened.  That needs a third
-    // ring stage: with two, loading tile j+1 waits for the release of tile
-    // j-1, which waits for the scores of tile j, i.e. for finish(j).
-    constexpr int LAG = (KF != kKeyBF16 && NST >= 3) ? 1 : 0;
-    for (int j = 0; j < n_kv + LAG; ++j) {
-      if (j < n_kv && !issue(j)) break;
-      const int jf = j - LAG;
-      if (jf >= 0 && relayed(jf) && !finish(jf)) break;
+    } else {
+      for (int j = 0; j < n_kv; ++j)
+        if (!issue(j)) break;
     }
+  } else if (warp >= 10) {
+    // ------------------------------------------------------------------ widening warps
+    // (quantised keys only): each widens half of every tile's codes
+    for (int j = 0; j < n_kv; ++j)
+      if (!finish(j, warp - 10, 2)) break;
   } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer
     {
@@ -458,10 +482,15 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
         // them into q . k (the scales arrived with the codes on c_full)
         const int st = j % NST;
         if (!__all_sync(0xffffffffu, mbar_wait(&c_full[st], (j / NST) & 1, p.err))) { ok = false; break; }
-        const float4* sc4 = reinterpret_cast<const float4*>(smem + C::OFF_SC + st * C::SCB);
+        const uint32_t sc_addr = smem_addr(smem + C::OFF_SC + st * C::SCB);
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          const float4 f = sc4[i];
+          // volatile loads keep the 32 scale vectors from all being hoisted
+          // ahead of their multiplies (128 more live registers: spills)
+          float4 f;
+          asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                       : "=f"(f.x), "=f"(f.y), "=f"(f.z), "=f"(f.w)
+                       : "r"(sc_addr + 16u * i));
           const float2 a = fmul2(make_float2(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1])),
                                  make_float2(f.x, f.y));
           const float2 c = fmul2(make_float2(__uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3])),
@@ -604,7 +633,7 @@ cudaError_t launch_t(const PrefillParams& p, cudaStream_t stream) {
   const long head_bytes = static_cast<long>(p.seq_lens ? p.kv_limit : p.S) * (R + DV) * 2;
   pp.head_group = static_cast<int>(std::max(1L, std::min<long>(p.B * p.Hq, (48L << 20) / head_bytes)));
   if (grid > 0x7fffffffL) return cudaErrorInvalidConfiguration;
-  kern<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(maps, pp);
+  kern<<<static_cast<unsigned>(grid), threads_for<KF>(), smem, stream>>>(maps, pp);
   return cudaGetLastError();
 }
 
