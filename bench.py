@@ -302,13 +302,14 @@ def measure_decode(rig, steps, warmup, mode="fused", min_seconds=0.0, info=None)
     return sec / steps
 
 
-def measure_decode_e2e(rig, steps):
+def measure_decode_e2e(rig, steps, graph=True):
     """Through host buffers and the public API: per step the step's query, new
     key and new value come from one page-locked host buffer (tk_copy_async,
     issued with the fused append + decode as one call prepared once, as a
-    serving loop with fixed buffers makes it), the kernel writes the output
-    straight into a page-locked host buffer (zero-copy), and the host
-    synchronises before the next step."""
+    serving loop with fixed buffers makes it; with graph=True the two are
+    recorded once as a CUDA graph and each step is one tk_graph_launch), the
+    kernel writes the output straight into a page-locked host buffer
+    (zero-copy), and the host synchronises before the next step."""
     torch = rig.torch
     tb = rig.tb
     hio = [c["io"].cpu().pin_memory() for c in rig.copies]
@@ -320,7 +321,8 @@ def measure_decode_e2e(rig, steps):
         B, hkv = cache.desc.batch, cache.desc.h_kv
         calls.append(tb.prepare_decode_append(cache, c["q"], c["k1"].view(B, hkv, -1),
                                               c["v1"].view(B, hkv, -1), c["seq_app"], rig.max_len,
-                                              ho, c["ws"], stream=stream, copy_in=(c["io"], h)))
+                                              ho, c["ws"], stream=stream, copy_in=(c["io"], h),
+                                              graph=graph))
     n = max(1, steps)
     for i in range(min(n, 20)):  # warm-up
         calls[i % len(calls)]()
@@ -783,7 +785,8 @@ def main():
     n = world
     value = n * rig.kv_bytes / sec_step / 1e9
     e2e_dt, h2d, d2h = measure_decode_e2e(rig, min(args.steps, 5000))
-    (e2e_dt,) = max_over_ranks(dist, (e2e_dt,), device)
+    e2e_eager_dt, _, _ = measure_decode_e2e(rig, min(args.steps, 2000), graph=False)
+    e2e_dt, e2e_eager_dt = max_over_ranks(dist, (e2e_dt, e2e_eager_dt), device)
     achieved = (rig.kv_bytes + rig.io_bytes) / sec_dec / 1e9
     dec_hash = source_hash("decode.cu", "common.cuh", "kv_row.cuh", "kernels.h")
     line = {
@@ -809,10 +812,13 @@ def main():
         "e2e": {"value": n * rig.kv_bytes / e2e_dt / 1e9, "unit": "GB/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_dt * 1e3,
+                "ms_per_step_without_graph": e2e_eager_dt * 1e3,
                 "how": "per step: the step's q, k_new, v_new from one page-locked host "
-                       "buffer (tk_copy_async) and the fused append + decode, issued as one "
-                       "prepared binding call; the kernel writes the output into page-locked "
-                       "host memory (zero-copy); host synchronisation every step"},
+                       "buffer (tk_copy_async) and the fused append + decode, prepared once "
+                       "by the binding and recorded as one CUDA graph (tk_graph_begin / "
+                       "tk_graph_end), replayed by one tk_graph_launch per step; the kernel "
+                       "writes the output into page-locked host memory (zero-copy); host "
+                       "synchronisation every step"},
         "gpu_launches": args.steps * timing.get("blocks", 1),
         "timing": {"blocks": timing.get("blocks"), "timed_region_s": timing.get("timed_region_s"),
                    "launches_per_step": 1,

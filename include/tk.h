@@ -58,7 +58,7 @@
 extern "C" {
 #endif
 
-#define TK_ABI_VERSION 2
+#define TK_ABI_VERSION 3
 
 typedef enum tk_status {
   TK_OK = 0,
@@ -286,6 +286,25 @@ tk_status tk_attn_decode_append(const tk_cache_desc* desc, const void* q, void* 
  * framework.  bytes == 0 is a no-op; NULL pointers give TK_ERR_INVALID_ARG,
  * a failed enqueue TK_ERR_CUDA.  Not part of the paper's method.            */
 tk_status tk_copy_async(void* dst, const void* src, size_t bytes, void* stream);
+
+/* CUDA-graph capture of a serving step, for loops that repeat the same calls
+ * on fixed buffers: tk_graph_begin starts capturing `stream` (relaxed mode,
+ * so the entry points' host-side set-up may run during the capture); every
+ * call enqueued on that stream until tk_graph_end (tk_copy_async, decode,
+ * append, prefill) is recorded instead of run; tk_graph_end stops the capture
+ * and returns an executable graph in *graph_out.  tk_graph_launch replays it
+ * on a stream (one launch for the whole step: far less host time per step
+ * than issuing each call); the replay uses the recorded pointers and sizes,
+ * so the contents of the buffers (queries, seq_lens, page table, host input
+ * buffer) may change between replays but not their addresses.
+ * tk_graph_destroy frees the graph.  Errors: NULL stream / graph pointers give
+ * TK_ERR_INVALID_ARG; a failed CUDA call gives TK_ERR_CUDA (a capture that
+ * fails inside tk_graph_end is ended and discarded).  Not part of the paper's
+ * method.                                                                    */
+tk_status tk_graph_begin(void* stream);
+tk_status tk_graph_end(void* stream, void** graph_out);
+tk_status tk_graph_launch(void* graph, void* stream);
+tk_status tk_graph_destroy(void* graph);
 
 /* Size of the fixed device scratch array used by tk_attn_decode_noalloc. */
 #define TK_DECODE_NOALLOC_SCRATCH_BYTES (8u << 20)

@@ -25,7 +25,8 @@ EXPORTED = ("tk_kv_append", "tk_attn_prefill", "tk_decode_workspace_size", "tk_a
             "tk_attn_decode_append", "tk_attn_decode_noalloc", "tk_attn_prefill_cached",
             "tk_attn_forward", "tk_backward_workspace_size", "tk_attn_backward", "tk_copy_async",
             "tk_check_wait_timeout", "tk_get_device_error", "tk_status_string", "tk_last_error",
-            "tk_abi_version")
+            "tk_abi_version", "tk_graph_begin", "tk_graph_end", "tk_graph_launch",
+            "tk_graph_destroy")
 
 
 class TkError(RuntimeError):
@@ -72,6 +73,10 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tk_get_device_error": (i32, [ctypes.POINTER(i32), vp]),
         "tk_check_wait_timeout": (i32, [i32, vp]),
         "tk_copy_async": (i32, [vp, vp, sz, vp]),
+        "tk_graph_begin": (i32, [vp]),
+        "tk_graph_end": (i32, [vp, ctypes.POINTER(vp)]),
+        "tk_graph_launch": (i32, [vp, vp]),
+        "tk_graph_destroy": (i32, [vp]),
         "tk_status_string": (ctypes.c_char_p, [i32]),
         "tk_last_error": (ctypes.c_char_p, []),
         "tk_abi_version": (i32, []),
@@ -344,18 +349,52 @@ class PreparedCall:
 
     For serving loops whose buffers stay fixed between steps: calling the
     object re-issues the same C calls in order (same pointers, same stream)
-    without the per-call Python checks, and raises TkError on a non-OK status."""
+    without the per-call Python checks, and raises TkError on a non-OK status.
+    With graph=True (a non-default stream required) the calls are run once,
+    then recorded once into a CUDA graph (tk_graph_begin / tk_graph_end), and
+    each call of the object is one tk_graph_launch of that graph."""
 
-    def __init__(self, name: str, args: tuple, keep: tuple, before: tuple = ()):
+    def __init__(self, name: str, args: tuple, keep: tuple, before: tuple = (), graph: bool = False,
+                 stream=None):
         L = load_library()
         self._calls = tuple((getattr(L, n), n, a) for n, a in (*before, (name, args)))
         self._keep = keep  # the tensors whose pointers are in args stay alive
+        self._graph = None
+        if graph:
+            if stream is None:
+                raise ValueError("graph=True needs a non-default stream")
+            self._stream = _stream(stream)
+            self._run_calls()                     # first run: checks and set-up outside capture
+            _check(L.tk_graph_begin(self._stream), "tk_graph_begin")
+            try:
+                self._run_calls()
+            finally:
+                g = ctypes.c_void_p()
+                st = L.tk_graph_end(self._stream, ctypes.byref(g))
+            _check(st, "tk_graph_end")
+            self._graph = g
+            self._launch = L.tk_graph_launch
+            self._destroy = L.tk_graph_destroy
 
-    def __call__(self):
+    def _run_calls(self):
         for fn, name, args in self._calls:
             st = fn(*args)
             if st != TK_OK:
                 _check(st, name)
+
+    def __call__(self):
+        if self._graph is not None:
+            st = self._launch(self._graph, self._stream)
+            if st != TK_OK:
+                _check(st, "tk_graph_launch")
+            return
+        self._run_calls()
+
+    def __del__(self):
+        g = getattr(self, "_graph", None)
+        if g is not None and g.value:
+            self._destroy(g)
+            self._graph = None
 
 
 def tk_copy_async(dst, src, stream=None):
@@ -372,13 +411,16 @@ def tk_copy_async(dst, src, stream=None):
 
 def prepare_decode_append(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_seq_len: int, out,
                           workspace, scale: float | None = None, stream=None,
-                          copy_in=None) -> PreparedCall:
+                          copy_in=None, graph: bool = False) -> PreparedCall:
     """tk_attn_decode_append with every argument checked once (see that function).
 
     copy_in = (dst, src): a device tensor and a page-locked host tensor of the
     same byte size, copied (tk_copy_async) before each decode -- e.g. the
     step's q, k_new and v_new packed in one host buffer.  `out` may be a
-    page-locked host tensor: the kernel then writes the result there directly."""
+    page-locked host tensor: the kernel then writes the result there directly.
+    graph=True records the step (copy and decode) as one CUDA graph launched
+    per call; preparing it runs the step twice (once eagerly, once recorded:
+    the recorded run does not execute), so the cache gets the new token once."""
     d = cache.desc
     dev = cache.k.device
     for t, n in ((q, "q"), (k_new, "k_new"), (v_new, "v_new")):
@@ -409,7 +451,8 @@ def prepare_decode_append(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_se
             _ptr(out), TK_F32 if out.dtype == torch.float32 else TK_BF16, ctypes.c_float(scale),
             _ptr(workspace), ctypes.c_size_t(workspace.numel()), _stream(stream))
     return PreparedCall("tk_attn_decode_append", args,
-                        (cache, q, k_new, v_new, seq_lens, out, workspace) + keep_in, before)
+                        (cache, q, k_new, v_new, seq_lens, out, workspace) + keep_in, before,
+                        graph=graph, stream=stream)
 
 
 def tk_attn_prefill(q, k, v, out, scale: float | None = None, causal: bool = True, stream=None):

@@ -446,6 +446,45 @@ tk_status tk_copy_async(void* dst, const void* src, size_t bytes, void* stream) 
   return TK_OK;
 }
 
+tk_status tk_graph_begin(void* stream) {
+  if (!stream) return fail(TK_ERR_INVALID_ARG, "graph capture needs a non-default stream");
+  const cudaError_t e = cudaStreamBeginCapture(static_cast<cudaStream_t>(stream),
+                                               cudaStreamCaptureModeRelaxed);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamBeginCapture");
+  return TK_OK;
+}
+
+tk_status tk_graph_end(void* stream, void** graph_out) {
+  if (!stream || !graph_out) return fail(TK_ERR_INVALID_ARG, "graph_end: NULL stream or graph_out");
+  *graph_out = nullptr;
+  cudaGraph_t g = nullptr;
+  cudaError_t e = cudaStreamEndCapture(static_cast<cudaStream_t>(stream), &g);
+  if (e != cudaSuccess) {
+    if (g) cudaGraphDestroy(g);
+    return cuda_fail(e, "cudaStreamEndCapture");
+  }
+  cudaGraphExec_t x = nullptr;
+  e = cudaGraphInstantiate(&x, g, 0);
+  cudaGraphDestroy(g);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGraphInstantiate");
+  *graph_out = x;
+  return TK_OK;
+}
+
+tk_status tk_graph_launch(void* graph, void* stream) {
+  if (!graph) return fail(TK_ERR_INVALID_ARG, "graph is NULL");
+  const cudaError_t e = cudaGraphLaunch(static_cast<cudaGraphExec_t>(graph), static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGraphLaunch");
+  return TK_OK;
+}
+
+tk_status tk_graph_destroy(void* graph) {
+  if (!graph) return fail(TK_ERR_INVALID_ARG, "graph is NULL");
+  const cudaError_t e = cudaGraphExecDestroy(static_cast<cudaGraphExec_t>(graph));
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGraphExecDestroy");
+  return TK_OK;
+}
+
 tk_status tk_check_wait_timeout(int32_t limit_us, void* stream) {
   if (limit_us < 1 || limit_us > 1000000)
     return fail(TK_ERR_INVALID_ARG, "limit_us=%d (1 .. 1000000)", limit_us);

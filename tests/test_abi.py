@@ -41,7 +41,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert tb.tk_abi_version() == 2
+    assert tb.tk_abi_version() == 3
     assert tb.tk_status_string(tb.TK_OK) == "TK_OK"
     assert tb.tk_status_string(tb.TK_ERR_WORKSPACE) == "TK_ERR_WORKSPACE"
     assert tb.tk_status_string(99) == "TK_ERR_UNKNOWN"
@@ -192,3 +192,14 @@ def test_wait_timeout_check_validation(lib):
     assert lib.tk_check_wait_timeout(0, None) == tb.TK_ERR_INVALID_ARG
     assert "limit_us" in tb.tk_last_error()
     assert lib.tk_check_wait_timeout(1000001, None) == tb.TK_ERR_INVALID_ARG
+
+
+def test_graph_entry_points_validate_before_cuda(lib):
+    """tk_graph_*: NULL streams / graphs are rejected before any CUDA call."""
+    g = ctypes.c_void_p()
+    assert lib.tk_graph_begin(None) == tb.TK_ERR_INVALID_ARG
+    assert lib.tk_graph_end(None, ctypes.byref(g)) == tb.TK_ERR_INVALID_ARG
+    assert lib.tk_graph_end(FAKE, None) == tb.TK_ERR_INVALID_ARG
+    assert lib.tk_graph_launch(None, None) == tb.TK_ERR_INVALID_ARG
+    assert lib.tk_graph_destroy(None) == tb.TK_ERR_INVALID_ARG
+

@@ -234,3 +234,38 @@ def test_prepared_call_with_host_input_and_zero_copy_output():
     with pytest.raises(ValueError):
         tb.prepare_decode_append(cache, qv, kv, vv, sl, 641, out_h, tb.decode_workspace(cache.desc, 641),
                                  copy_in=(io, hio[:-1]))
+
+
+def test_prepared_call_as_cuda_graph():
+    """graph=True: the copy-in and the fused decode recorded as one CUDA graph; each
+    replay takes the host buffer's current contents and gives the eager call's bits."""
+    require_gpu()
+    B, hq, hkv, r, dv = 4, 32, 8, 32, 128
+    lens = [100, 640, 1, 300]
+    cache, _, _ = _make(B, hq, hkv, r, dv, lens, False, 0, seed=71)
+    other = _clone(cache)
+    sl = torch.tensor(lens, dtype=torch.int32, device="cuda")
+    io = torch.empty(B * hq * r + B * hkv * (r + dv), dtype=torch.bfloat16, device="cuda")
+    nq, nk = B * hq * r, B * hkv * r
+    qv, kv, vv = io[:nq].view(B, hq, r), io[nq:nq + nk].view(B, hkv, r), io[nq + nk:].view(B, hkv, dv)
+    hio = torch.empty(io.numel(), dtype=torch.bfloat16).pin_memory()
+    out_h = torch.full((B, hq, dv), float("nan")).pin_memory()
+    stream = torch.cuda.Stream()
+    ws = tb.decode_workspace(cache.desc, 641)
+    for step, seed in enumerate((72, 82)):
+        q = inputs.normal_bf16((B, hq, r), seed=seed, device="cuda")
+        k1 = inputs.normal_bf16((B, hkv, r), seed=seed + 1, device="cuda")
+        v1 = inputs.normal_bf16((B, hkv, dv), seed=seed + 2, device="cuda")
+        hio.copy_(torch.cat([q.flatten(), k1.flatten(), v1.flatten()]).cpu())
+        if step == 0:   # preparing runs the step once eagerly, then records it
+            call = tb.prepare_decode_append(cache, qv, kv, vv, sl, 641, out_h, ws, stream=stream,
+                                            copy_in=(io, hio), graph=True)
+        call()
+        stream.synchronize()
+        assert tb.tk_get_device_error() == 0
+        out_d = torch.empty(B, hq, dv, device="cuda")
+        tb.tk_attn_decode_append(other, q, k1, v1, sl, 641, out_d, tb.decode_workspace(other.desc, 641))
+        torch.cuda.synchronize()
+        assert torch.equal(out_h, out_d.cpu())
+        _same_cache(other, cache)
+    del call
