@@ -64,6 +64,30 @@ def quantize_int4_per_token(k) -> tuple[np.ndarray, np.ndarray]:
     return codes, scale
 
 
+def quantize_int4_per_group(k, group: int) -> tuple[np.ndarray, np.ndarray]:
+    """Quantise keys [..., r] to int4 codes with one fp32 scale per `group`
+    consecutive channels (r a multiple of group): scales [..., r // group].
+    Each group is quantised exactly as quantize_int4_per_token quantises a
+    whole row (amax / 7, binary32 division, ties to even); with group == r
+    the two coincide.  Used to measure what the coarser one-scale-per-token
+    reading costs in accuracy; the kernels store one scale per token."""
+    k32 = np.asarray(k, dtype=np.float32)
+    r = k32.shape[-1]
+    if r % group:
+        raise ValueError(f"r={r} is not a multiple of group={group}")
+    g = k32.reshape(*k32.shape[:-1], r // group, group)
+    codes, scales = quantize_int4_per_token(g)
+    return codes.reshape(k32.shape), scales
+
+
+def dequantize_per_group(codes, scales) -> np.ndarray:
+    """codes [..., r] times the scale of each channel's group (scales [..., r // group]), in fp64."""
+    c = np.asarray(codes, dtype=np.float64)
+    s = np.asarray(scales, dtype=np.float64)
+    group = c.shape[-1] // s.shape[-1]
+    return c * np.repeat(s, group, axis=-1)
+
+
 def pack_int4(codes) -> np.ndarray:
     """int4 codes [..., r] (r even, values in [-8, 7]) -> bytes [..., r/2]:
     element 2j in bits 0-3, element 2j+1 in bits 4-7."""

@@ -473,3 +473,53 @@ def test_append_contiguous_and_paged_agree():
     with pytest.raises(ValueError):
         oc.append_contiguous(np.zeros((1, 1, 4, 2)), np.zeros((1, 1, 4, 2)), [3],
                              np.zeros((1, 1, 2, 2)), np.zeros((1, 1, 2, 2)))
+
+
+# ---------------------------------------------------------------- int4 scale grouping
+
+def test_int4_per_group_reduces_to_per_token_and_is_groupwise():
+    """One group spanning the row is the per-token quantiser; smaller groups
+    quantise each group on its own (a group's codes ignore the other groups)."""
+    rng = np.random.default_rng(31)
+    k = rng.standard_normal((3, 5, 64)).astype(np.float32)
+    c_tok, s_tok = oc.quantize_int4_per_token(k)
+    c_g, s_g = oc.quantize_int4_per_group(k, 64)
+    assert np.array_equal(c_g, c_tok) and np.array_equal(s_g[..., 0], s_tok)
+    c32, s32 = oc.quantize_int4_per_group(k, 32)
+    assert s32.shape == (3, 5, 2)
+    for h in range(2):
+        ch, sh = oc.quantize_int4_per_token(k[..., 32 * h:32 * h + 32])
+        assert np.array_equal(c32[..., 32 * h:32 * h + 32], ch) and np.array_equal(s32[..., h], sh)
+    # dequantised error within half a step of each channel's own group scale
+    err = np.abs(oc.dequantize_per_group(c32, s32) - k)
+    assert np.all(err <= np.repeat(s32, 32, axis=-1) / 2 + 1e-7)
+    with pytest.raises(ValueError):
+        oc.quantize_int4_per_group(k, 48)
+
+
+def int4_grouping_errors(r, group, seed=0, n_q=64, n_k=2048, dv=64):
+    """Mean relative error (sum|out - ref| / sum|ref|) of decode attention over int4 keys,
+    one scale per token vs one per `group` channels, against the unquantised keys."""
+    rng = np.random.default_rng(seed)
+    q = rng.standard_normal((n_q, r))
+    k = rng.standard_normal((n_k, r)).astype(np.float32)
+    v = rng.standard_normal((n_k, dv))
+    scale = 1 / math.sqrt(r)
+    ref = oa.attention_head(q, k.astype(np.float64), v, scale)
+    c_t, s_t = oc.quantize_int4_per_token(k)
+    c_g, s_g = oc.quantize_int4_per_group(k, group)
+    out_t = oa.attention_head(q, oa.dequantize_keys(c_t, s_t), v, scale)
+    out_g = oa.attention_head(q, oc.dequantize_per_group(c_g, s_g), v, scale)
+    rel = lambda o: float(np.abs(o - ref).sum() / np.abs(ref).sum())
+    return rel(out_t), rel(out_g)
+
+
+@pytest.mark.parametrize("r", [64, 128])
+def test_int4_per_token_scale_costs_little_accuracy(r):
+    """The library stores one fp32 scale per token.  Groups of 32 channels would cut
+    the attention error (the largest |k| of 32 channels is smaller than of r), at the
+    price of r / 32 scales per token; measured here on N(0,1) keys and queries."""
+    e_tok, e_grp = int4_grouping_errors(r, 32, seed=r)
+    print(f"\n[int4 scale grouping] r={r}: mean rel error per token {e_tok:.4f}, "
+          f"per 32 channels {e_grp:.4f} (ratio {e_tok / e_grp:.2f})")
+    assert e_grp < e_tok < 2.0 * e_grp
