@@ -153,3 +153,36 @@ def test_quantised_key_decode_r_sweep(kfmt, r):
                                      1 / math.sqrt(r)))
         got.append(f64(out[b, g * G:(g + 1) * G]))
     parity(np.concatenate(got), np.concatenate(ref), what=f"{kfmt} keys r={r}, full size")
+
+
+# ------------------------------------------------------------------ GPT-2-small layer
+
+def test_gpt2_small_layer_prefill_then_32_decode_steps():
+    """The GPT-2-small-shaped layer as the benchmark runs it: causal prefill of 256
+    tokens (fp32 out), the prompt appended, then 32 fused append + decode steps;
+    every output element of every step against the oracle."""
+    require_gpu()
+    B, H, r, dv, S, T = 1, 12, 16, 64, 256, 32
+    scale = 1 / math.sqrt(r)
+    q = inputs.normal_bf16((B, H, S, r), 2001, device="cuda")
+    k = inputs.normal_bf16((B, H, S, r), 2002, device="cuda")
+    v = inputs.normal_bf16((B, H, S, dv), 2003, device="cuda")
+    pre = torch.empty(B, H, S, dv, device="cuda")
+    tb.tk_attn_prefill(q, k, v, pre)
+    parity(f64(pre), oa.attention_prefill(f64(q), f64(k), f64(v), scale), what="gpt2 layer prefill")
+    cache = tb.ThinKeyCache.allocate(B, H, H, r, dv, capacity=S + T)
+    tb.tk_kv_append(cache, k, v, torch.zeros(B, dtype=torch.int32, device="cuda"))
+    ws = tb.decode_workspace(cache.desc, S + T)
+    kk, vv = f64(k)[0], f64(v)[0]
+    for t in range(T):
+        qd = inputs.normal_bf16((B, H, r), 2100 + 3 * t, device="cuda")
+        k1 = inputs.normal_bf16((B, H, r), 2101 + 3 * t, device="cuda")
+        v1 = inputs.normal_bf16((B, H, dv), 2102 + 3 * t, device="cuda")
+        out = torch.empty(B, H, dv, device="cuda")
+        sl = torch.full((B,), S + t, dtype=torch.int32, device="cuda")
+        tb.tk_attn_decode_append(cache, qd, k1, v1, sl, S + T, out, ws)
+        kk = np.concatenate([kk, f64(k1)[0][:, None]], axis=1)
+        vv = np.concatenate([vv, f64(v1)[0][:, None]], axis=1)
+        ref = oa.attention_decode(f64(qd), kk[None], vv[None], [S + t + 1], scale)
+        parity(f64(out), ref, what=f"gpt2 layer decode step {t}")
+    assert tb.tk_get_device_error() == 0
