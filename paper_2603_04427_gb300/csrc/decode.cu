@@ -497,49 +497,10 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.k)) : "memory");
       asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.v)) : "memory");
     }
-    if (p.fuse_append && u_begin < u_end) {
-      // Append fused into the decode: the CTA that reads the last chunk of a
-      // (b, g) pair first writes that pair's new token at position
-      // seq_lens[b] (exactly as the append kernel does), then orders the
-      // writes before its own TMA reads of the chunk with a proxy fence.  No
-      // other CTA reads that chunk.
-      Walker wk;
-      wk.seek(u_begin, pre, lens, B, Hkv);
-      while (true) {
-        const long long last = wk.cp + wk.nb - 1;
-        if (last >= u_end) break;  // this pair's last chunk belongs to a later CTA
-        const int pos = wk.Lb - 1;
-        if (p.seq_lens[wk.b] == pos) {  // not clamped: the new token fits
-          long long row = -1;
-          if (ps == 0) {
-            row = (static_cast<long long>(wk.b) * Hkv + wk.g) * p.capacity + pos;
-          } else {
-            const int page = p.page_table[static_cast<long long>(wk.b) * p.max_pages + (pos >> p.page_shift)];
-            if (page >= 0 && page < p.num_pages)
-              row = (static_cast<long long>(page) * Hkv + wk.g) * ps + (pos & (ps - 1));
-            else if (lane == 0)
-              record_error(p.err, TK_DEVERR_INDEX);
-          }
-          if (row >= 0) {
-            const long long src = static_cast<long long>(wk.b) * Hkv + wk.g;
-            write_kv_row<R, DV, KF>(const_cast<void*>(p.k), const_cast<void*>(p.v),
-                                     const_cast<float*>(p.k_scale), static_cast<size_t>(row),
-                                     static_cast<const unsigned char*>(p.k_new) + src * 2 * R,
-                                     static_cast<const unsigned char*>(p.v_new) + src * 2 * DV, lane);
-          }
-        }
-        if (last + 1 >= u_end) break;
-        wk.chunk = wk.nb - 1;
-        wk.next(pre, lens, Hkv);
-      }
-      asm volatile("fence.proxy.async.global;" ::: "memory");
-      __syncwarp();
-      asm volatile("fence.proxy.async.global;" ::: "memory");
-    }
     bool ok = true;
     for (long long w0 = u_begin; ok && w0 < u_end; w0 += 32) {
       // lane j prepares unit w0 + j: first cache row of the chunk, valid tokens, query offset
-      long long row = 0;
+      long long row = 0, app = -1;
       int n = 0, qoff = 0, g = 0, b = 0, t0 = 0;
       const long long u = w0 + lane;
       if (u < u_end) {
@@ -549,6 +510,22 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
         t0 = wk.chunk * kChunk;
         n = min(kChunk, wk.Lb - t0);
         qoff = (b * p.Hq + g * G) * R;
+        // Append fused into the decode: the chunk holding a pair's last token gets
+        // the step's new token written at position seq_lens[b] (exactly as the
+        // append kernel does) just before its TMA loads are issued; no other CTA
+        // reads that chunk.  A clamped length (the token does not fit) gets no write.
+        if (p.fuse_append && wk.chunk + 1 == wk.nb && p.seq_lens[b] == wk.Lb - 1) {
+          const int pos = wk.Lb - 1;
+          if (ps == 0) {
+            app = (static_cast<long long>(b) * Hkv + g) * p.capacity + pos;
+          } else {
+            const int page = p.page_table[static_cast<long long>(b) * p.max_pages + (pos >> p.page_shift)];
+            if (page >= 0 && page < p.num_pages)
+              app = (static_cast<long long>(page) * Hkv + g) * ps + (pos & (ps - 1));
+            else
+              record_error(p.err, TK_DEVERR_INDEX);
+          }
+        }
         if (ps == 0) {
           row = (static_cast<long long>(b) * Hkv + g) * p.capacity + t0;
         } else {
@@ -568,6 +545,18 @@ decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
         const int bj = __shfl_sync(0xffffffffu, b, j);
         const int gj = __shfl_sync(0xffffffffu, g, j);
         const int tj = __shfl_sync(0xffffffffu, t0, j);
+        const long long aj = __shfl_sync(0xffffffffu, app, j);
+        if (aj >= 0) {
+          // the new row, then a proxy fence: the TMA reads below see it
+          const long long src = static_cast<long long>(bj) * Hkv + gj;
+          write_kv_row<R, DV, KF>(const_cast<void*>(p.k), const_cast<void*>(p.v),
+                                   const_cast<float*>(p.k_scale), static_cast<size_t>(aj),
+                                   static_cast<const unsigned char*>(p.k_new) + src * 2 * R,
+                                   static_cast<const unsigned char*>(p.v_new) + src * 2 * DV, lane);
+          asm volatile("fence.proxy.async.global;" ::: "memory");
+          __syncwarp();
+          asm volatile("fence.proxy.async.global;" ::: "memory");
+        }
         if (lane == 0) {
           const long long i = w0 + j - u_begin;
           const int st = static_cast<int>(i % C::NSTAGE);
