@@ -714,8 +714,8 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--headline-only", action="store_true",
                     help="skip the secondary workloads and the CPU baseline")
-    ap.add_argument("--only", choices=("prefill", "chunked", "backward", "gpt2", "paged", "int8",
-                                       "cpu"),
+    ap.add_argument("--only", choices=("decode", "prefill", "chunked", "backward", "gpt2", "paged",
+                                       "int8", "cpu"),
                     help="run one secondary workload alone (for profiling) and print its result; "
                          "cpu: the oracle's time on every workload")
     args = ap.parse_args()
@@ -758,6 +758,12 @@ def main():
                 res[kf] = measure_chunked_prefill(wl.CHUNKED_PREFILL, args.steps, device, torch, k_fmt=kf)
         elif args.only == "gpt2":
             res.update(measure_gpt2_layer(wl.GPT2_LAYER, args.steps, device, torch))
+        elif args.only == "decode":
+            # the headline workload's decode kernel alone (tk_attn_decode), for profiling
+            drig = DecodeRig(w, device)
+            sd = measure_decode(drig, args.steps, args.warmup, mode="decode")
+            res.update(decode_kernel_us=sd * 1e6, kv_bytes=drig.kv_bytes,
+                       frac=(drig.kv_bytes + drig.io_bytes) / sd / 1e9 / peaks["hbm_gbs"])
         else:
             ow = wl.PAGED_LONG_DECODE if args.only == "paged" else wl.INT8_DECODE
             orig = DecodeRig(ow, device, copies=1)
@@ -788,7 +794,7 @@ def main():
     e2e_eager_dt, _, _ = measure_decode_e2e(rig, min(args.steps, 2000), graph=False)
     e2e_dt, e2e_eager_dt = max_over_ranks(dist, (e2e_dt, e2e_eager_dt), device)
     achieved = (rig.kv_bytes + rig.io_bytes) / sec_dec / 1e9
-    dec_hash = source_hash("decode.cu", "common.cuh", "kv_row.cuh", "kernels.h")
+    dec_hash = source_hash("decode.cu", "common.cuh", "kv_row.cuh", "kernels.h", "widen.cuh")
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": n, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": sec_step * 1e3, "higher_is_better": True,
@@ -899,7 +905,8 @@ def main():
                                  "frac": r3(pf["tflops"] / peaks["bf16_tflops"]),
                                  "peak_source": peak_src,
                                  "traffic": recorded_traffic("prefill", pw.name, source_hash(
-                                     "prefill.cu", "common.cuh", "tc05.cuh"))})
+                                     "prefill.cu", "common.cuh", "tc05.cuh", "widen.cuh",
+                                     "kernels.h"))})
         else:
             pre.update(pf)
         if n == 1:
