@@ -412,8 +412,10 @@ __device__ void prefetch_first_chunks(const DecodeParams& p, int lane, int limit
 }
 
 
+// The grid is persistent (CTAS_PER_SM CTAs on every SM at once): the bound
+// keeps the register count low enough for that many CTAs to be resident.
 template <int R, int DV, int G, int KF>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, Cfg<R, DV, G, KF>::CTAS_PER_SM)
 decode_kernel(const __grid_constant__ DecodeMaps maps, const DecodeParams p) {
   using C = Cfg<R, DV, G, KF>;
   constexpr bool KI8 = KF != 0;  // quantised keys (int8 or int4)
