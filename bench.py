@@ -373,8 +373,9 @@ def measure_prefill(w, iters, device, torch):
 
 def measure_chunked_prefill(w, iters, device, torch, k_fmt="bf16"):
     """A prompt chunk of w.seq tokens after w.cached cached ones: tk_attn_prefill_cached
-    (append of the chunk + attention over the cache), bf16 output; keys stored as
-    bf16, int8 or int4.  The append launch is also timed on its own."""
+    (append of the chunk, for int8 / int4 keys the widening of the context's keys into
+    the workspace, attention over the cache), bf16 output; keys stored as bf16, int8 or
+    int4.  The append launch is also timed on its own."""
     from paper_2603_04427_gb300 import binding as tb
     from paper_2603_04427_gb300 import cost_model as cm
     from paper_2603_04427_gb300 import inputs
@@ -389,9 +390,10 @@ def measure_chunked_prefill(w, iters, device, torch, k_fmt="bf16"):
     vn = inputs.normal_bf16((B, hkv, S, dv), w.seed + 5, device=device)
     out = torch.empty(B, hq, S, dv, dtype=torch.bfloat16, device=device)
     sl = torch.full((B,), L0, dtype=torch.int32, device=device)
+    ws = tb.prefill_cached_workspace(cache, L0 + S)
 
     def enq(_):  # the same chunk re-appended at the same positions every time
-        tb.tk_attn_prefill_cached(cache, q, kn, vn, sl, L0 + S, out)
+        tb.tk_attn_prefill_cached(cache, q, kn, vn, sl, L0 + S, out, workspace=ws)
 
     def enq_append(_):
         tb.tk_kv_append(cache, kn, vn, sl)
@@ -400,7 +402,8 @@ def measure_chunked_prefill(w, iters, device, torch, k_fmt="bf16"):
     sec_app = graph_time(torch, enq_append, iters, 3, max_graph=16, min_seconds=0.1) / iters
     flops = cm.prefill_flops(B, hq, S, r, dv, cached=L0)
     return {"ms": sec * 1e3, "tflops": flops / sec / 1e12, "flops_per_call": flops,
-            "cached": L0, "launches": 2, "append_ms": sec_app * 1e3, "k_dtype": k_fmt}
+            "cached": L0, "launches": 2 if k_fmt == "bf16" else 3, "append_ms": sec_app * 1e3,
+            "k_dtype": k_fmt}
 
 
 def measure_backward(w, iters, device, torch):

@@ -58,7 +58,7 @@
 extern "C" {
 #endif
 
-#define TK_ABI_VERSION 3
+#define TK_ABI_VERSION 4
 
 typedef enum tk_status {
   TK_OK = 0,
@@ -201,20 +201,36 @@ tk_status tk_attn_backward(const void* q, const void* k, const void* v, const vo
  *              modified; the caller advances it by seq afterwards)
  *   max_seq_len: host bound of seq_lens[b] + seq
  *   out      : device [batch][h_q][seq][d_v], TK_BF16 or TK_F32
+ *   workspace: int8 / int4 keys: device scratch of
+ *              tk_prefill_cached_workspace_size(desc, max_seq_len) bytes,
+ *              256-byte aligned (else TK_ERR_WORKSPACE); unused (may be
+ *              NULL) for bf16 keys.  Overwritten by every call; reusable by
+ *              later calls in stream order.
  * Keys of every k_dtype (Section 6: thin keys compose with key
- * quantisation): the products run on the tensor cores from bf16 tiles, int8
- * and int4 codes widened to bf16 exactly in shared memory, and each score
- * q . code multiplied by its key's fp32 scale.  Contiguous or paged caches;
- * a sequence whose chunk does not fit sets the device error word and is
- * computed over a clamped context.  Cache slots past a sequence's context
- * may hold anything (they are never weighted).  seq_lens[b] == 0 gives the
- * plain causal prefill of the chunk.  Two launches (append, then attention)
- * in stream order.                                                        */
+ * quantisation): the products run on the tensor cores from bf16 tiles.
+ * int8 / int4 keys are first widened, once per token of each context, into
+ * the workspace: for r <= 64 each key scale * code becomes two bf16 terms
+ * hi + lo (within 2^-17 of it, relative) and S = Q hi^T + Q lo^T; for
+ * r = 128 the codes become exact bf16 and each score q . code is multiplied
+ * by its key's fp32 scale.  Contiguous or paged caches; a sequence whose
+ * chunk does not fit sets the device error word and is computed over a
+ * clamped context.  Cache slots past a sequence's context may hold anything
+ * (they are never weighted).  seq_lens[b] == 0 gives the plain causal
+ * prefill of the chunk.  Launches in stream order: append, (key widening,)
+ * attention.                                                              */
 tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void* k_cache,
                                  void* v_cache, float* k_scale, const int32_t* page_table,
                                  const int32_t* seq_lens, const void* k_new, const void* v_new,
                                  int32_t seq, int32_t max_seq_len, void* out, int32_t out_dtype,
-                                 float scale, int32_t causal, void* stream);
+                                 float scale, int32_t causal, void* workspace,
+                                 size_t workspace_bytes, void* stream);
+
+/* Bytes of workspace tk_attn_prefill_cached needs for a cache of this shape
+ * and this bound of seq_lens[b] + seq: two bf16 planes of r per token and kv
+ * head (r <= 64), or one plane and one fp32 scale per token (r = 128), over
+ * min(max_seq_len, the cache's tokens per sequence) rows rounded up to a
+ * multiple of 4.  0 for bf16 keys or an invalid descriptor.              */
+size_t tk_prefill_cached_workspace_size(const tk_cache_desc* desc, int32_t max_seq_len);
 
 /* Bytes of decode workspace needed for a cache of this shape when no
  * sequence is longer than max_seq_len, on the current device (the split of

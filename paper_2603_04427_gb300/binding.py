@@ -23,6 +23,7 @@ LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtk.so")
 
 EXPORTED = ("tk_kv_append", "tk_attn_prefill", "tk_decode_workspace_size", "tk_attn_decode",
             "tk_attn_decode_append", "tk_attn_decode_noalloc", "tk_attn_prefill_cached",
+            "tk_prefill_cached_workspace_size",
             "tk_attn_forward", "tk_backward_workspace_size", "tk_attn_backward", "tk_copy_async",
             "tk_check_wait_timeout", "tk_get_device_error", "tk_status_string", "tk_last_error",
             "tk_abi_version", "tk_graph_begin", "tk_graph_end", "tk_graph_launch",
@@ -65,7 +66,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tk_attn_backward": (i32, [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, i32, i32, i32, i32,
                                    i32, i32, f32, i32, vp]),
         "tk_attn_prefill_cached": (i32, [dp, vp, vp, vp, vp, vp, vp, vp, vp, i32, i32, vp, i32,
-                                         f32, i32, vp]),
+                                         f32, i32, vp, sz, vp]),
+        "tk_prefill_cached_workspace_size": (sz, [dp, i32]),
         "tk_attn_decode": (i32, [dp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp, sz, vp]),
         "tk_attn_decode_append": (i32, [dp, vp, vp, vp, vp, vp, vp, vp, vp, i32, vp, i32, f32, vp,
                                         sz, vp]),
@@ -315,11 +317,20 @@ def tk_attn_backward(q, k, v, out, d_out, lse, dq, dk, dv, workspace=None,
     return dq, dk, dv
 
 
+def prefill_cached_workspace(cache: ThinKeyCache, max_seq_len: int):
+    """The device workspace tk_attn_prefill_cached needs for this cache and this
+    bound of seq_lens[b] + S (int8 / int4 keys), or None (bf16 keys)."""
+    n = int(load_library().tk_prefill_cached_workspace_size(ctypes.byref(cache.desc), int(max_seq_len)))
+    return torch.empty(n, dtype=torch.uint8, device=cache.k.device) if n else None
+
+
 def tk_attn_prefill_cached(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_seq_len: int, out,
-                           scale: float | None = None, causal: bool = True, stream=None):
+                           scale: float | None = None, causal: bool = True, workspace=None,
+                           stream=None):
     """Append a chunk (k_new [B, H_kv, S, r], v_new [B, H_kv, S, d_v] bf16) at seq_lens[b]
     and prefill its queries q [B, H_q, S, r] over the cache (query i at position
-    seq_lens[b] + i) -> out [B, H_q, S, d_v] (fp32 or bf16).  bf16, int8 or int4 keys."""
+    seq_lens[b] + i) -> out [B, H_q, S, d_v] (fp32 or bf16).  bf16, int8 or int4 keys;
+    quantised keys need a workspace (prefill_cached_workspace; allocated here if None)."""
     d = cache.desc
     dev = cache.k.device
     for t, n in ((q, "q"), (k_new, "k_new"), (v_new, "v_new")):
@@ -335,12 +346,18 @@ def tk_attn_prefill_cached(cache: ThinKeyCache, q, k_new, v_new, seq_lens, max_s
         raise ValueError("q / k_new / v_new / out shapes do not match the cache")
     scale = 1.0 / math.sqrt(d.r) if scale is None else float(scale)
     L = load_library()
+    if workspace is None and d.k_dtype != TK_BF16:
+        workspace = prefill_cached_workspace(cache, max_seq_len)
+    if workspace is not None:
+        _need(workspace, torch.uint8, "workspace", dev)
     _check(L.tk_attn_prefill_cached(ctypes.byref(d), _ptr(q), _ptr(cache.k), _ptr(cache.v),
                                     _ptr(cache.k_scale), _ptr(cache.page_table), _ptr(seq_lens),
                                     _ptr(k_new), _ptr(v_new),
                                     S, int(max_seq_len), _ptr(out),
                                     TK_F32 if out.dtype == torch.float32 else TK_BF16, scale,
-                                    1 if causal else 0, _stream(stream)), "tk_attn_prefill_cached")
+                                    1 if causal else 0, _ptr(workspace),
+                                    0 if workspace is None else workspace.numel(),
+                                    _stream(stream)), "tk_attn_prefill_cached")
     return out
 
 

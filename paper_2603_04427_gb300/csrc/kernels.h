@@ -103,6 +103,13 @@ struct PrefillParams {
   int k_fmt;                // cache keys: 0 bf16, 1 int8, 2 int4 (cached mode only)
   const float* k_scale;     // fp32 per-token key scales (int8 / int4 keys)
   float* lse;               // optional [B][Hq][S]: natural-log logsumexp of each row's scores
+  // int8 / int4 keys: device workspace the context's keys are widened into
+  // (prefill_workspace_bytes(B, Hkv, R, DV, k_fmt, kw_rows) bytes, 256-byte
+  // aligned), kw_rows >= kv_limit rows per (b, kv head), a multiple of 4
+  void* kw;
+  size_t kw_bytes;
+  int kw_rows;
+  const float* kw_scale;    // set by the launcher: the workspace's scale plane, if any
 };
 
 struct BackwardParams {
@@ -132,6 +139,9 @@ cudaError_t launch_backward(const BackwardParams& p, cudaStream_t stream, int* u
 // The tensor-memory gradient kernel, after the preprocessing pass.
 cudaError_t launch_backward_tc(const BackwardParams& p, cudaStream_t stream, int* unsupported);
 
+// Bytes of workspace the prefill of a quantised-key cache needs (0 for bf16
+// keys or an unsupported shape).
+size_t prefill_workspace_bytes(int B, int Hkv, int R, int DV, int k_fmt, int rows);
 cudaError_t launch_prefill(const PrefillParams& p, cudaStream_t stream, int* unsupported);
 
 // One thread waits limit_ns on an mbarrier that nothing arrives at, through the

@@ -19,8 +19,15 @@
 //     read S from TMEM, apply the causal / length mask, keep the running max m
 //     and sum l (log2 domain), write P = exp2(S * scale*log2e - m) as bf16 into
 //     the first 64 TMEM columns of S, and at the end write O / l.
-//   warps 10-11 (int8 / int4 key caches only): widen each K tile's codes to
-//     bf16 in the swizzled operand layout, half a tile each.
+// int8 / int4 key caches: key_widen_kernel first widens the context's keys
+// once into a contiguous workspace, which the TMA warp then loads like bf16
+// keys.  Where shared memory holds two K tiles per stage (r <= 64) each key
+// becomes scale * code as the two-term bf16 sum hi + lo
+// (|hi + lo - scale * code| <= 2^-17 |scale * code|) and S takes 2r/16 MMA
+// steps, Q against hi and then against lo, so the softmax is that of bf16
+// keys; otherwise (r = 128) the workspace holds the codes as exact bf16 with
+// the fp32 scales beside them, and the softmax multiplies each score by its
+// key's scale.
 // The running max is updated lazily: O and l are rescaled only when a tile's
 // maximum exceeds the max in use by more than 8 (a factor 256), so the
 // weights stay <= 256 and the result is unchanged (O / l uses one consistent
@@ -41,9 +48,6 @@ namespace {
 constexpr int kBM = 128;          // query rows per tile
 constexpr int kBN = 128;          // keys per kv tile
 constexpr int kThreads = 320;     // 2 x 4 softmax warps, 1 TMA warp, 1 MMA warp
-// quantised-key caches add two warps that widen the key codes of each tile
-template <int KF>
-constexpr int threads_for() { return KF == 0 ? kThreads : kThreads + 64; }
 constexpr int kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 // P of a tile is published in kParts key ranges, so the P V products of one
@@ -95,23 +99,20 @@ struct PCfg {
   static constexpr int VB = kBN * DV * 2;
   static constexpr int V_NBOX = DV / 64;             // 128-byte-wide boxes of V
   static constexpr int V_BOXB = kBN * 128;
-  // quantised keys: a tile's codes (r or r/2 bytes per key) land in a staging
-  // area of the stage, and its 128 fp32 key scales after them
-  static constexpr int CODE_ROWB = KF == kKeyInt8 ? R : (KF == kKeyInt4 ? R / 2 : 0);
-  static constexpr int STGB = kBN * CODE_ROWB;
-  static constexpr int SCB = KF == kKeyBF16 ? 0 : kBN * 4;
   static constexpr int QBA = (QB + 1023) / 1024 * 1024;  // one Q tile, 1 KB aligned
   static constexpr int OFF_Q = 0;                        // two Q tiles
   static constexpr int OFF_K = 2 * QBA;
   static constexpr int KBA = (KB + 1023) / 1024 * 1024;
-  static constexpr int STAGE = KBA + VB;
-  static constexpr int NST = (2 * QBA + 3 * (STAGE + SCB) + 2 * STGB + 2048 <= 200 * 1024) ? 3 : 2;
-  // raw codes wait in a staging slot until the widening warps have widened
-  // them: one slot per stage where shared memory allows, else two slots that
-  // the TMA warp reuses once they are free; the scales keep one slot per stage
-  static constexpr int NSTG = (2 * QBA + NST * (STAGE + SCB + STGB) + 2048 <= 200 * 1024) ? NST : 2;
-  static constexpr int OFF_STG = OFF_K + NST * STAGE;
-  static constexpr int OFF_SC = OFF_STG + NSTG * STGB;
+  // K tiles per stage: 2 for quantised keys widened to hi + lo (where two
+  // stages of them fit), else 1 (bf16 keys, or exact bf16 codes whose scales
+  // the softmax applies)
+  static constexpr int KT = (KF != 0 && 2 * QBA + 2 * (2 * KBA + VB) + 2048 <= 200 * 1024) ? 2 : 1;
+  static constexpr bool SCALE_IN_SOFTMAX = KF != 0 && KT == 1;
+  static constexpr int SCB = SCALE_IN_SOFTMAX ? kBN * 4 : 0;  // a tile's key scales
+  static constexpr int VOFF = KT * KBA;              // V tile offset in a stage
+  static constexpr int STAGE = VOFF + VB;
+  static constexpr int NST = (2 * QBA + 3 * (STAGE + SCB) + 2048 <= 200 * 1024) ? 3 : 2;
+  static constexpr int OFF_SC = OFF_K + NST * STAGE;
   static constexpr int OFF_BAR = OFF_SC + NST * SCB;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;      // + slack to align the base to 1 KB
   static_assert(SMEM <= 227 * 1024, "shared memory");
@@ -119,19 +120,54 @@ struct PCfg {
   static constexpr uint32_t IDESC_O = instr_desc(kBM, DV, true);
 };
 
-// Byte offset, inside a K tile, of the 16-byte piece holding elements e0 .. e0+7
-// (e0 a multiple of 8) of key `row`, in the layout the TMA writes with the
-// tile's swizzle: box e0 / QK_BOX, row pitch QK_SW bytes, and the piece's index
-// within its row XORed with address bits 7.. (32-, 64- or 128-byte swizzle).
-template <class C>
-__device__ __forceinline__ uint32_t k_piece_offset(int row, int e0) {
-  const uint32_t o = static_cast<uint32_t>(row * C::QK_SW + (e0 % C::QK_BOX) * 2);
-  constexpr uint32_t mask = static_cast<uint32_t>(C::QK_SW / 16 - 1) << 4;
-  return static_cast<uint32_t>((e0 / C::QK_BOX) * C::QK_BOXB) + (o ^ ((o >> 3) & mask));
+// Exact fp32 values of four int8 codes: each code, biased by 128, becomes the
+// low byte of the float 2^23 + (c + 128), and 2^23 + 128 is subtracted.
+__device__ __forceinline__ void i8x4_to_f32(uint32_t w, float2& a, float2& b) {
+  const uint32_t x = w ^ 0x80808080u;
+  uint32_t f0, f1, f2, f3;
+  asm("prmt.b32 %0, %1, 0x4B000000, 0x7540;" : "=r"(f0) : "r"(x));
+  asm("prmt.b32 %0, %1, 0x4B000000, 0x7541;" : "=r"(f1) : "r"(x));
+  asm("prmt.b32 %0, %1, 0x4B000000, 0x7542;" : "=r"(f2) : "r"(x));
+  asm("prmt.b32 %0, %1, 0x4B000000, 0x7543;" : "=r"(f3) : "r"(x));
+  const float2 bias = make_float2(-8388736.0f, -8388736.0f);  // -(2^23 + 128)
+  a = fadd2(make_float2(__uint_as_float(f0), __uint_as_float(f1)), bias);
+  b = fadd2(make_float2(__uint_as_float(f2), __uint_as_float(f3)), bias);
+}
+
+// Exact fp32 values of eight int4 codes (element 2i in the low nibble of byte
+// i, 2i+1 in its high nibble, 4-bit two's complement): c + 8 = nibble ^ 8
+// becomes the low byte of 2^23 + (c + 8), and 2^23 + 8 is subtracted.
+__device__ __forceinline__ void i4x8_to_f32(uint32_t w, float2 (&o)[4]) {
+  const uint32_t t = w ^ 0x88888888u;
+  const uint32_t lo = t & 0x0F0F0F0Fu, hi = (t >> 4) & 0x0F0F0F0Fu;
+  const float2 bias = make_float2(-8388616.0f, -8388616.0f);  // -(2^23 + 8)
+  uint32_t a[4], b[4];
+  asm("prmt.b32 %0, %1, 0x4B000000, 0x7540;" : "=r"(a[0]) : "r"(lo));
+  asm("prmt.b32 %0, %1, 0x4B000000, 0x7541;" : "=r"(a[1]) : "r"(lo));
+  asm("prmt.b32 %0, %1, 0x4B000000, 0x7542;" : "=r"(a[2]) : "r"(lo));
+  asm("prmt.b32 %0, %1, 0x4B000000, 0x7543;" : "=r"(a[3]) : "r"(lo));
+  asm("prmt.b32 %0, %1, 0x4B000000, 0x7540;" : "=r"(b[0]) : "r"(hi));
+  asm("prmt.b32 %0, %1, 0x4B000000, 0x7541;" : "=r"(b[1]) : "r"(hi));
+  asm("prmt.b32 %0, %1, 0x4B000000, 0x7542;" : "=r"(b[2]) : "r"(hi));
+  asm("prmt.b32 %0, %1, 0x4B000000, 0x7543;" : "=r"(b[3]) : "r"(hi));
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    o[i] = fadd2(make_float2(__uint_as_float(a[i]), __uint_as_float(b[i])), bias);
+}
+
+// x as two bf16 pairs with hi + lo = x to within 2^-17 |x|: hi = bf16(x), and
+// x - hi (exact in fp32) rounded to bf16.  Low halves hold x.x.
+__device__ __forceinline__ void split_bf16(float2 x, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(x.x, x.y);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  const float2 d = fadd2(x, make_float2(-__uint_as_float(hi << 16), -__uint_as_float(hi & 0xffff0000u)));
+  const __nv_bfloat162 l = __floats2bfloat162_rn(d.x, d.y);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 
 struct Maps {
   CUtensorMap q, k, v;
+  CUtensorMap klo;  // lo plane of widened quantised keys (two K tiles per stage)
 };
 
 // One CTA (one per SM) computes two consecutive 128-row query tiles, A and B,
@@ -146,7 +182,7 @@ struct Maps {
 //   warp 8: TMA producer (Q tiles once, K/V tiles into an NST-stage ring)
 //   warp 9: MMA issuer
 template <int R, int DV, int KF>
-__global__ void __launch_bounds__(threads_for<KF>(), 1)
+__global__ void __launch_bounds__(kThreads, 1)
 prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   using C = PCfg<R, DV, KF>;
   constexpr int NST = C::NST;
@@ -161,9 +197,9 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   uint64_t* s_full = kv_empty + NST;            // [2] (tile A, tile B)
   uint64_t* p_full = s_full + 2;                // [tile][part]: P of one key range
   uint64_t* o_full = p_full + 2 * kParts;       // [2]
-  uint64_t* c_full = o_full + 2;                // [NST] cached mode: raw K tile (+ scales) landed
-  uint64_t* stg_free = c_full + NST;            // [NSTG] quantised keys: staging slot widened
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(stg_free + C::NSTG);
+  uint64_t* c_full = o_full + 2;                // [NST] cached mode: the last tile landed
+  uint64_t* sc_full = c_full + NST;             // [NST] key scales landed (scales in the softmax)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sc_full + NST);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int n_qt = (p.S + kBM - 1) / kBM;
@@ -203,13 +239,12 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   if (tid == 0) {
     mbar_init(q_full, 1);
     for (int s = 0; s < NST; ++s) {
-      // quantised keys: both widening warps arrive on k_full; otherwise the TMA warp
-      mbar_init(&k_full[s], KF == kKeyBF16 ? 1 : 2);
+      mbar_init(&k_full[s], 1);
       mbar_init(&v_full[s], 1);
       mbar_init(&kv_empty[s], 1);
       mbar_init(&c_full[s], 1);
+      mbar_init(&sc_full[s], 1);
     }
-    for (int s = 0; s < C::NSTG; ++s) mbar_init(&stg_free[s], 2);
     for (int x = 0; x < 2; ++x) {
       mbar_init(&s_full[x], 1);
       for (int h = 0; h < kParts; ++h) mbar_init(&p_full[kParts * x + h], 128);
@@ -225,64 +260,27 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  // A tile is "relayed" when it must be finished in shared memory before the MMA
-  // warp may read it: every tile of a quantised cache (codes widened to bf16,
-  // by the two widening warps) and, in cached mode, the tile holding the
-  // context's end (value rows past it zeroed by the TMA warp: the cache may hold
-  // anything there, and 0 * NaN would spread).  Other tiles go straight from the
-  // TMA to k_full.
+  // In cached mode the tile holding the context's end is "relayed": it lands on
+  // c_full, the TMA warp zeroes its value rows past the context (the cache may
+  // hold anything there, and 0 * NaN would spread) and then publishes it on
+  // k_full.  Other tiles go straight from the TMA to k_full.
   const bool relay = p.seq_lens != nullptr;
-  auto relayed = [&](int j) {
-    return relay && (KF != kKeyBF16 || kv_len - j * kBN < kBN);
-  };
-  // finish(j, part, nparts) of a relayed tile, by warp `part` of the nparts
-  // warps that share it: widen its share of the codes, zero its share of the
-  // value rows past the context, then publish on k_full (nparts arrivals)
-  auto finish = [&](int j, int part, int nparts) -> bool {
+  auto relayed = [&](int j) { return relay && kv_len - j * kBN < kBN; };
+  auto finish = [&](int j) -> bool {
     const int st = j % NST;
-    unsigned char* sk = smem + C::OFF_K + st * C::STAGE;
-    unsigned char* sv = sk + C::KBA;
-    // quantised caches use c_full on every tile; a bf16 cache only on its last
-    const uint32_t phc = KF != kKeyBF16 ? (j / NST) & 1 : 0;
-    bool okc = mbar_wait(&c_full[st], phc, p.err);
-    const int n_valid = kv_len - j * kBN;
-    if (n_valid < kBN) okc = mbar_wait(&v_full[st], (j / NST) & 1, p.err) && okc;
+    unsigned char* sv = smem + C::OFF_K + st * C::STAGE + C::VOFF;
+    const bool okc = mbar_wait(&c_full[st], 0, p.err) && mbar_wait(&v_full[st], (j / NST) & 1, p.err);
     if (!__all_sync(0xffffffffu, okc)) return false;
-    if constexpr (KF != kKeyBF16) {
-      const unsigned char* stg = smem + C::OFF_STG + (j % C::NSTG) * C::STGB;
-      constexpr int PPR = R / 8;  // 16-byte bf16 pieces per key row
-#pragma unroll 4
-      for (int c = part * 32 + lane; c < kBN * PPR; c += 32 * nparts) {
-        const int row = c / PPR, e0 = (c % PPR) * 8;
-        // exact widening by integer moves (no int-to-float conversions, which
-        // would share the ex2 unit with the softmax warps)
-        uint4 o;
-        if constexpr (KF == kKeyInt8) {
-          const uint2 w = *reinterpret_cast<const uint2*>(stg + row * C::CODE_ROWB + e0);
-          i8x4_to_bf16(w.x, o.x, o.y);
-          i8x4_to_bf16(w.y, o.z, o.w);
-        } else {
-          const uint32_t w = *reinterpret_cast<const uint32_t*>(stg + row * C::CODE_ROWB + e0 / 2);
-          i4x8_to_bf16(w, o.x, o.y, o.z, o.w);
-        }
-        *reinterpret_cast<uint4*>(sk + k_piece_offset<C>(row, e0)) = o;
-      }
-    }
-    if (n_valid < kBN) {
-      const int first = max(n_valid, 0);
-      const int per_box = (kBN - first) * 8;   // 16-byte pieces per value box
-      for (int c = part * 32 + lane; c < per_box * C::V_NBOX; c += 32 * nparts) {
-        const int box = c / per_box, rem2 = c % per_box;
-        *reinterpret_cast<uint4*>(sv + box * C::V_BOXB + (first + rem2 / 8) * 128 + (rem2 % 8) * 16) =
-            make_uint4(0u, 0u, 0u, 0u);
-      }
+    const int first = max(kv_len - j * kBN, 0);
+    const int per_box = (kBN - first) * 8;   // 16-byte pieces per value box
+    for (int c = lane; c < per_box * C::V_NBOX; c += 32) {
+      const int box = c / per_box, rem2 = c % per_box;
+      *reinterpret_cast<uint4*>(sv + box * C::V_BOXB + (first + rem2 / 8) * 128 + (rem2 % 8) * 16) =
+          make_uint4(0u, 0u, 0u, 0u);
     }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     __syncwarp();
-    if (lane == 0) {
-      mbar_arrive(&k_full[st]);
-      if constexpr (KF != kKeyBF16) mbar_arrive(&stg_free[j % C::NSTG]);  // staging slot read
-    }
+    if (lane == 0) mbar_arrive(&k_full[st]);
     return true;
   };
 
@@ -309,9 +307,6 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       const int st = j % NST;
       int okw = 1;
       if (j >= NST && lane == 0) okw = mbar_wait(&kv_empty[st], ((j / NST) - 1) & 1, p.err);
-      // quantised keys: staging slot j % NSTG must have been widened (tile j - NSTG)
-      if (KF != kKeyBF16 && j >= C::NSTG && lane == 0 && okw)
-        okw = mbar_wait(&stg_free[j % C::NSTG], ((j / C::NSTG) - 1) & 1, p.err);
       if (!__shfl_sync(0xffffffffu, okw, 0)) return false;
       // lane s < nsub finds the plane and first row of sub-box s
       int plane = kv_plane, row = j * kBN;
@@ -336,39 +331,28 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       }
       if (lane == 0) {
         unsigned char* sk = smem + C::OFF_K + st * C::STAGE;
-        unsigned char* sv = sk + C::KBA;
+        unsigned char* sv = sk + C::VOFF;
+        uint64_t* kb = relayed(j) ? &c_full[st] : &k_full[st];
         if constexpr (KF == kKeyBF16) {
-          uint64_t* kb = relayed(j) ? &c_full[st] : &k_full[st];
           mbar_arrive_expect_tx(kb, C::KB);
           for (int s2 = 0; s2 < nsub; ++s2)
             for (int i = 0; i < C::QK_NBOX; ++i)
               tma_load_3d(sk + i * C::QK_BOXB + s2 * bps * C::QK_SW, &maps.k, i * C::QK_BOX,
                           rows[s2], planes[s2], kb);
         } else {
-          // raw codes into staging slot j % NSTG (emptied by the widening warps,
-          // waited for above), the tile's key scales into the stage's slot
-          unsigned char* stg = smem + C::OFF_STG + (j % C::NSTG) * C::STGB;
-          float* sc = reinterpret_cast<float*>(smem + C::OFF_SC + st * C::SCB);
-          const int kv0 = j * kBN;
-          uint32_t sc_bytes = 0;
-          if (p.page_size == 0) {
-            sc_bytes = static_cast<uint32_t>(min(kBN, p.capacity - kv0)) * 4u;
-          } else {
-            for (int s2 = 0; s2 < nsub; ++s2)
-              if (planes[s2] >= 0) sc_bytes += static_cast<uint32_t>(bps) * 4u;
+          // widened keys from the workspace: [B*Hkv][kw_rows][r] planes, one box per tile
+          mbar_arrive_expect_tx(kb, C::KT * C::KB);
+          for (int i = 0; i < C::QK_NBOX; ++i) {
+            tma_load_3d(sk + i * C::QK_BOXB, &maps.k, i * C::QK_BOX, j * kBN, kv_plane, kb);
+            if constexpr (C::KT == 2)
+              tma_load_3d(sk + C::KBA + i * C::QK_BOXB, &maps.klo, i * C::QK_BOX, j * kBN, kv_plane, kb);
           }
-          mbar_arrive_expect_tx(&c_full[st], static_cast<uint32_t>(nsub * bps * C::CODE_ROWB) + sc_bytes);
-          for (int s2 = 0; s2 < nsub; ++s2)
-            tma_load_3d(stg + s2 * bps * C::CODE_ROWB, &maps.k, 0, rows[s2], planes[s2], &c_full[st]);
-          if (p.page_size == 0) {
-            bulk_g2s(sc, p.k_scale + static_cast<size_t>(kv_plane) * p.capacity + kv0, sc_bytes,
-                     &c_full[st]);
-          } else {
-            for (int s2 = 0; s2 < nsub; ++s2)
-              if (planes[s2] >= 0)
-                bulk_g2s(sc + s2 * bps,
-                         p.k_scale + static_cast<size_t>(planes[s2]) * p.page_size + rows[s2],
-                         static_cast<uint32_t>(bps) * 4u, &c_full[st]);
+          if constexpr (C::SCALE_IN_SOFTMAX) {
+            // the tile's key scales (rows past kw_rows are never weighted)
+            const uint32_t bytes = static_cast<uint32_t>(min(kBN, p.kw_rows - j * kBN)) * 4u;
+            mbar_arrive_expect_tx(&sc_full[st], bytes);
+            bulk_g2s(smem + C::OFF_SC + st * C::SCB,
+                     p.kw_scale + static_cast<size_t>(kv_plane) * p.kw_rows + j * kBN, bytes, &sc_full[st]);
           }
         }
         mbar_arrive_expect_tx(&v_full[st], C::VB);
@@ -379,20 +363,10 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       }
       return true;
     };
-    if constexpr (KF == kKeyBF16) {
-      for (int j = 0; j < n_kv; ++j) {
-        if (!issue(j)) break;
-        if (relayed(j) && !finish(j, 0, 1)) break;
-      }
-    } else {
-      for (int j = 0; j < n_kv; ++j)
-        if (!issue(j)) break;
+    for (int j = 0; j < n_kv; ++j) {
+      if (!issue(j)) break;
+      if (relayed(j) && !finish(j)) break;
     }
-  } else if (warp >= 10) {
-    // ------------------------------------------------------------------ widening warps
-    // (quantised keys only): each widens half of every tile's codes
-    for (int j = 0; j < n_kv; ++j)
-      if (!finish(j, warp - 10, 2)) break;
   } else if (warp == 9) {
     // ------------------------------------------------------------------ MMA issuer
     {
@@ -400,13 +374,20 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       // stages and K steps are start-address offsets from these
       const Desc dq = make_desc(smem_addr(smem + C::OFF_Q), 16, 8 * C::QK_SW, C::QK_LAYOUT);
       const Desc dk = make_desc(smem_addr(smem + C::OFF_K), 16, 8 * C::QK_SW, C::QK_LAYOUT);
-      const Desc dv = make_desc(smem_addr(smem + C::OFF_K + C::KBA), C::V_BOXB, 1024, 2u);
+      const Desc dv = make_desc(smem_addr(smem + C::OFF_K + C::VOFF), C::V_BOXB, 1024, 2u);
       auto issue_s = [&](int x, int st) {  // S_x = Q_x K^T
         const uint32_t qo = x * C::QBA, ko = st * C::STAGE;
 #pragma unroll
         for (int k = 0; k < R / 16; ++k) {
           const uint32_t off = (k / C::KSTEP_PER_BOX) * C::QK_BOXB + (k % C::KSTEP_PER_BOX) * 32;
           mma_ss_e(tmem + x * 128, dq.at(qo + off), dk.at(ko + off), C::IDESC_S, k > 0);
+        }
+        if constexpr (C::KT == 2) {  // + Q_x lo^T
+#pragma unroll
+          for (int k = 0; k < R / 16; ++k) {
+            const uint32_t off = (k / C::KSTEP_PER_BOX) * C::QK_BOXB + (k % C::KSTEP_PER_BOX) * 32;
+            mma_ss_e(tmem + x * 128, dq.at(qo + off), dk.at(ko + C::KBA + off), C::IDESC_S, 1u);
+          }
         }
         tc_commit_e(&s_full[x]);
       };
@@ -477,11 +458,11 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       // the whole S row of this thread: 128 fp32 scores
       uint32_t v[128];
       tmem_ld128(tS + lane_off, v);
-      if constexpr (KF != kKeyBF16) {
+      if constexpr (C::SCALE_IN_SOFTMAX) {
         // quantised keys: the products are q . code; each key's fp32 scale turns
-        // them into q . k (the scales arrived with the codes on c_full)
+        // them into q . k (the scales arrive on sc_full)
         const int st = j % NST;
-        if (!__all_sync(0xffffffffu, mbar_wait(&c_full[st], (j / NST) & 1, p.err))) { ok = false; break; }
+        if (!__all_sync(0xffffffffu, mbar_wait(&sc_full[st], (j / NST) & 1, p.err))) { ok = false; break; }
         const uint32_t sc_addr = smem_addr(smem + C::OFF_SC + st * C::SCB);
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
@@ -599,6 +580,76 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
   }
 }
 
+// Widens the keys of each sequence's context, tokens 0 .. seq_lens[b] + S - 1
+// of an int8 / int4 cache (contiguous or paged), into the workspace planes
+// [B*Hkv][kw_rows][r] that the prefill loads by TMA: hi and lo of
+// scale * code (KT = 2), or the codes as exact bf16 with the fp32 scales in
+// sc[B*Hkv][kw_rows] (KT = 1).  Once per token, where widening inside the
+// prefill would redo it for every query tile pair that reads the tile.  One
+// thread per 8 elements of one token; rows past a context are left as they
+// are (their scores are masked and their value rows zeroed).
+template <int R, int KF, int KT>
+__global__ void __launch_bounds__(256) key_widen_kernel(const PrefillParams p, __nv_bfloat16* hi,
+                                                        __nv_bfloat16* lo, float* sc) {
+  constexpr int PPR = R / 8;
+  const long long i = static_cast<long long>(blockIdx.x) * 256 + threadIdx.x;
+  if (i >= static_cast<long long>(p.B) * p.Hkv * p.kw_rows * PPR) return;
+  const int piece = static_cast<int>(i % PPR);
+  const long long tok = i / PPR;
+  const int t = static_cast<int>(tok % p.kw_rows);
+  const int plane = static_cast<int>(tok / p.kw_rows);  // b * Hkv + g
+  const int b = plane / p.Hkv, g = plane - b * p.Hkv;
+  // seq_lens[b] clamped as the prefill kernel clamps it (and records the error)
+  const int L0 = min(max(p.seq_lens[b], 0), p.kv_limit - p.S);
+  if (t >= L0 + p.S) return;
+  long long row;  // cache row of token t
+  if (p.page_size == 0) {
+    row = static_cast<long long>(plane) * p.capacity + t;
+  } else {
+    int page = p.page_table[static_cast<long long>(b) * p.max_pages + (t >> p.page_shift)];
+    if (page < 0 || page >= p.num_pages) {
+      record_error(p.err, TK_DEVERR_INDEX);
+      page = 0;
+    }
+    row = (static_cast<long long>(page) * p.Hkv + g) * p.page_size + (t & (p.page_size - 1));
+  }
+  const float s = p.k_scale[row];
+  const size_t o = static_cast<size_t>(tok) * R + piece * 8;
+  if constexpr (KT == 2) {
+    float2 x[4];
+    if constexpr (KF == kKeyInt8) {
+      const uint2 w = *reinterpret_cast<const uint2*>(static_cast<const int8_t*>(p.k) + row * R + piece * 8);
+      i8x4_to_f32(w.x, x[0], x[1]);
+      i8x4_to_f32(w.y, x[2], x[3]);
+    } else {
+      i4x8_to_f32(*reinterpret_cast<const uint32_t*>(static_cast<const uint8_t*>(p.k) + row * (R / 2) +
+                                                     piece * 4),
+                  x);
+    }
+    const float2 s2 = make_float2(s, s);
+    uint4 h, l;
+    split_bf16(fmul2(x[0], s2), h.x, l.x);
+    split_bf16(fmul2(x[1], s2), h.y, l.y);
+    split_bf16(fmul2(x[2], s2), h.z, l.z);
+    split_bf16(fmul2(x[3], s2), h.w, l.w);
+    *reinterpret_cast<uint4*>(hi + o) = h;
+    *reinterpret_cast<uint4*>(lo + o) = l;
+  } else {
+    uint4 h;
+    if constexpr (KF == kKeyInt8) {
+      const uint2 w = *reinterpret_cast<const uint2*>(static_cast<const int8_t*>(p.k) + row * R + piece * 8);
+      i8x4_to_bf16(w.x, h.x, h.y);
+      i8x4_to_bf16(w.y, h.z, h.w);
+    } else {
+      i4x8_to_bf16(*reinterpret_cast<const uint32_t*>(static_cast<const uint8_t*>(p.k) + row * (R / 2) +
+                                                      piece * 4),
+                   h.x, h.y, h.z, h.w);
+    }
+    *reinterpret_cast<uint4*>(hi + o) = h;
+    if (piece == 0) sc[tok] = s;
+  }
+}
+
 // ---------------------------------------------------------------- host side
 
 template <int R, int DV, int KF>
@@ -615,12 +666,27 @@ cudaError_t launch_t(const PrefillParams& p, cudaStream_t stream) {
     kv_planes = p.num_pages * p.Hkv;
     box_rows = std::min(p.page_size, kBN);
   }
+  PrefillParams pp = p;
   bool ok = make_map(&maps.q, p.q, R, p.S, p.B * p.Hq, C::QK_BOX, kBM, C::QK_SW) &&
             make_map(&maps.v, p.v, DV, kv_rows, kv_planes, 64, box_rows, 128);
-  if constexpr (KF == kKeyBF16)
+  __nv_bfloat16 *hi = nullptr, *lo = nullptr;
+  float* sc = nullptr;
+  if constexpr (KF == kKeyBF16) {
     ok = ok && make_map(&maps.k, p.k, R, kv_rows, kv_planes, C::QK_BOX, box_rows, C::QK_SW);
-  else  // rows of codes, copied as they are into the staging area
-    ok = ok && make_map_bytes(&maps.k, p.k, C::CODE_ROWB, kv_rows, kv_planes, box_rows);
+  } else {
+    // workspace: plane 0 = hi (or the bf16 codes), then lo (or the scales)
+    if (!p.kw || p.kw_bytes < prefill_workspace_bytes(p.B, p.Hkv, R, DV, KF, p.kw_rows) ||
+        p.kw_rows % 4 != 0 || p.kw_rows < p.kv_limit)
+      return cudaErrorInvalidValue;
+    const size_t plane = static_cast<size_t>(p.B) * p.Hkv * p.kw_rows * R;
+    hi = static_cast<__nv_bfloat16*>(p.kw);
+    if constexpr (C::KT == 2) lo = hi + plane;
+    else sc = reinterpret_cast<float*>(hi + plane);
+    pp.kw_scale = sc;
+    ok = ok && make_map(&maps.k, hi, R, p.kw_rows, p.B * p.Hkv, C::QK_BOX, kBN, C::QK_SW);
+    if constexpr (C::KT == 2)
+      ok = ok && make_map(&maps.klo, lo, R, p.kw_rows, p.B * p.Hkv, C::QK_BOX, kBN, C::QK_SW);
+  }
   if (!ok) return cudaErrorInvalidValue;
   auto kern = prefill_kernel<R, DV, KF>;
   const int smem = C::SMEM;
@@ -628,12 +694,16 @@ cudaError_t launch_t(const PrefillParams& p, cudaStream_t stream) {
   if (e != cudaSuccess) return e;
   const long n_qt = (p.S + kBM - 1) / kBM;
   const long grid = (n_qt + 1) / 2 * p.B * p.Hq;  // one CTA per query tile pair
-  PrefillParams pp = p;
+  if (grid > 0x7fffffffL) return cudaErrorInvalidConfiguration;
+  if constexpr (KF != kKeyBF16) {
+    const long long n = static_cast<long long>(p.B) * p.Hkv * p.kw_rows * (R / 8);
+    key_widen_kernel<R, KF, C::KT><<<static_cast<unsigned>((n + 255) / 256), 256, 0, stream>>>(p, hi, lo, sc);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
   // about 48 MB of K/V per head group
   const long head_bytes = static_cast<long>(p.seq_lens ? p.kv_limit : p.S) * (R + DV) * 2;
   pp.head_group = static_cast<int>(std::max(1L, std::min<long>(p.B * p.Hq, (48L << 20) / head_bytes)));
-  if (grid > 0x7fffffffL) return cudaErrorInvalidConfiguration;
-  kern<<<static_cast<unsigned>(grid), threads_for<KF>(), smem, stream>>>(maps, pp);
+  kern<<<static_cast<unsigned>(grid), kThreads, smem, stream>>>(maps, pp);
   return cudaGetLastError();
 }
 
@@ -664,6 +734,29 @@ cudaError_t by_dv(const PrefillParams& p, cudaStream_t s, int* uns) {
 }
 
 }  // namespace
+
+template <int R, int DV>
+size_t ws_bytes_t(int B, int Hkv, int k_fmt, int rows) {
+  const size_t plane = static_cast<size_t>(B) * Hkv * rows * R * 2;  // bf16 [B*Hkv][rows][r]
+  bool two = PCfg<R, DV, kKeyInt8>::KT == 2;
+  if constexpr (R >= 32) {
+    if (k_fmt == kKeyInt4) two = PCfg<R, DV, kKeyInt4>::KT == 2;
+  } else {
+    if (k_fmt == kKeyInt4) return 0;  // int4 keys need r >= 32
+  }
+  return two ? 2 * plane : plane + static_cast<size_t>(B) * Hkv * rows * 4;
+}
+
+size_t prefill_workspace_bytes(int B, int Hkv, int R, int DV, int k_fmt, int rows) {
+  if (k_fmt == kKeyBF16 || B <= 0 || Hkv <= 0 || rows <= 0 || (DV != 64 && DV != 128)) return 0;
+  switch (R) {
+    case 16: return DV == 64 ? ws_bytes_t<16, 64>(B, Hkv, k_fmt, rows) : ws_bytes_t<16, 128>(B, Hkv, k_fmt, rows);
+    case 32: return DV == 64 ? ws_bytes_t<32, 64>(B, Hkv, k_fmt, rows) : ws_bytes_t<32, 128>(B, Hkv, k_fmt, rows);
+    case 64: return DV == 64 ? ws_bytes_t<64, 64>(B, Hkv, k_fmt, rows) : ws_bytes_t<64, 128>(B, Hkv, k_fmt, rows);
+    case 128: return DV == 64 ? ws_bytes_t<128, 64>(B, Hkv, k_fmt, rows) : ws_bytes_t<128, 128>(B, Hkv, k_fmt, rows);
+  }
+  return 0;
+}
 
 cudaError_t launch_prefill(const PrefillParams& p, cudaStream_t stream, int* unsupported) {
   *unsupported = 0;

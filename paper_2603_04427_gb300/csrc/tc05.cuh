@@ -259,21 +259,4 @@ inline bool make_map(CUtensorMap* m, const void* base, int inner, int rows, int 
              CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// 3-D map over [planes][rows][row_bytes] bytes (int8 / packed int4 key codes),
-// no swizzle, a (row_bytes x box_rows x 1) box; row_bytes a multiple of 16.
-inline bool make_map_bytes(CUtensorMap* m, const void* base, int row_bytes, int rows, int planes,
-                           int box_rows) {
-  auto enc = encode_fn();
-  if (!enc) return false;
-  cuuint64_t dims[3] = {static_cast<cuuint64_t>(row_bytes), static_cast<cuuint64_t>(rows),
-                        static_cast<cuuint64_t>(planes)};
-  cuuint64_t strides[2] = {static_cast<cuuint64_t>(row_bytes),
-                           static_cast<cuuint64_t>(row_bytes) * rows};
-  cuuint32_t box[3] = {static_cast<cuuint32_t>(row_bytes), static_cast<cuuint32_t>(box_rows), 1};
-  cuuint32_t estr[3] = {1, 1, 1};
-  return enc(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<void*>(base), dims, strides, box, estr,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 }  // namespace tk

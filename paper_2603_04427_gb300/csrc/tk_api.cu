@@ -262,11 +262,21 @@ tk_status prefill_impl(const void* q, const void* k, const void* v, void* out, f
 }
 }  // namespace
 
+namespace {
+// Rows per (b, kv head) of the prefill's widened-key workspace: the bound of
+// seq_lens[b] + seq within the cache, rounded up to a multiple of 4.
+int prefill_kw_rows(const tk_cache_desc* d, int32_t max_seq_len) {
+  const int cache_tokens = d->page_size ? d->max_pages_per_seq * d->page_size : d->capacity;
+  return (std::min(max_seq_len, cache_tokens) + 3) / 4 * 4;
+}
+}  // namespace
+
 tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void* k_cache,
                                  void* v_cache, float* k_scale, const int32_t* page_table,
                                  const int32_t* seq_lens, const void* k_new, const void* v_new,
                                  int32_t seq, int32_t max_seq_len, void* out, int32_t out_dtype,
-                                 float scale, int32_t causal, void* stream) {
+                                 float scale, int32_t causal, void* workspace,
+                                 size_t workspace_bytes, void* stream) {
   tk_status s = check_desc(desc);
   if (s != TK_OK) return s;
   if (seq < 0 || max_seq_len < seq)
@@ -281,12 +291,29 @@ tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void*
     return fail(TK_ERR_INVALID_ARG, "q / out / seq_lens / k_new / v_new is NULL");
   if (!aligned16(q) || !aligned16(out) || !aligned16(k_new) || !aligned16(v_new))
     return fail(TK_ERR_INVALID_ARG, "q / out / k_new / v_new must be 16-byte aligned");
+  const int cache_tokens = desc->page_size ? desc->max_pages_per_seq * desc->page_size
+                                           : desc->capacity;
+  const int kv_limit = std::min(max_seq_len, cache_tokens);
+  if (kv_limit < seq)
+    return fail(TK_ERR_INVALID_ARG, "seq=%d does not fit the cache (%d tokens)", seq, kv_limit);
+  const bool quant = desc->k_dtype != TK_BF16;
+  const int kw_rows = quant ? prefill_kw_rows(desc, max_seq_len) : 0;
+  if (quant) {
+    const size_t need = tk::prefill_workspace_bytes(desc->batch, desc->h_kv, desc->r, desc->d_v,
+                                                    key_format(desc->k_dtype), kw_rows);
+    if (need == 0)
+      return fail(TK_ERR_UNSUPPORTED, "prefill: no kernel for r=%d d_v=%d k_dtype=%d", desc->r,
+                  desc->d_v, desc->k_dtype);
+    if (!workspace || reinterpret_cast<uintptr_t>(workspace) % 256 != 0)
+      return fail(TK_ERR_WORKSPACE, "workspace is NULL or not 256-byte aligned");
+    if (workspace_bytes < need)
+      return fail(TK_ERR_WORKSPACE, "workspace has %zu bytes, %zu needed", workspace_bytes, need);
+  }
   DeviceInfo dev;
   if ((s = device_info(&dev)) != TK_OK) return s;
   const cudaStream_t st = static_cast<cudaStream_t>(stream);
   // 1. the chunk's keys and values into the cache at seq_lens[b]
   tk::AppendParams a{};
-  const bool quant = desc->k_dtype != TK_BF16;
   a.k = k_cache; a.v = v_cache; a.k_scale = quant ? k_scale : nullptr; a.page_table = page_table;
   a.seq_lens = seq_lens; a.k_new = k_new; a.v_new = v_new; a.err = dev.err;
   a.B = desc->batch; a.Hkv = desc->h_kv; a.R = desc->r; a.DV = desc->d_v; a.T = seq;
@@ -317,15 +344,20 @@ tk_status tk_attn_prefill_cached(const tk_cache_desc* desc, const void* q, void*
   p.page_shift = a.page_shift;
   p.num_pages = desc->num_pages;
   p.max_pages = desc->max_pages_per_seq;
-  const int cache_tokens = desc->page_size ? desc->max_pages_per_seq * desc->page_size
-                                           : desc->capacity;
-  p.kv_limit = std::min(max_seq_len, cache_tokens);
-  if (p.kv_limit < seq)
-    return fail(TK_ERR_INVALID_ARG, "seq=%d does not fit the cache (%d tokens)", seq, p.kv_limit);
+  p.kv_limit = kv_limit;
+  p.kw = quant ? workspace : nullptr;
+  p.kw_bytes = quant ? workspace_bytes : 0;
+  p.kw_rows = kw_rows;
   e = tk::launch_prefill(p, st, &uns);
   if (uns) return fail(TK_ERR_UNSUPPORTED, "prefill: no kernel for r=%d d_v=%d", desc->r, desc->d_v);
   if (e != cudaSuccess) return cuda_fail(e, "prefill launch");
   return TK_OK;
+}
+
+size_t tk_prefill_cached_workspace_size(const tk_cache_desc* desc, int32_t max_seq_len) {
+  if (check_desc(desc) != TK_OK || max_seq_len <= 0 || desc->k_dtype == TK_BF16) return 0;
+  return tk::prefill_workspace_bytes(desc->batch, desc->h_kv, desc->r, desc->d_v,
+                                     key_format(desc->k_dtype), prefill_kw_rows(desc, max_seq_len));
 }
 
 size_t tk_decode_workspace_size(const tk_cache_desc* desc, int32_t max_seq_len) {

@@ -41,7 +41,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_abi_version_and_status_strings(lib):
-    assert tb.tk_abi_version() == 3
+    assert tb.tk_abi_version() == 4
     assert tb.tk_status_string(tb.TK_OK) == "TK_OK"
     assert tb.tk_status_string(tb.TK_ERR_WORKSPACE) == "TK_ERR_WORKSPACE"
     assert tb.tk_status_string(99) == "TK_ERR_UNKNOWN"
@@ -131,16 +131,47 @@ def test_prefill_cached_validation(lib):
     d8 = _desc(k_dtype=tb.TK_I8)
     # int8 keys need their scales
     assert P(ctypes.byref(d8), FAKE, FAKE, FAKE, None, None, FAKE, FAKE, FAKE, 64, 256, FAKE,
-             tb.TK_BF16, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG
+             tb.TK_BF16, 0.1, 1, None, 0, None) == tb.TK_ERR_INVALID_ARG
     assert "k_scale" in tb.tk_last_error()
     assert P(ctypes.byref(d), FAKE, FAKE, FAKE, None, None, FAKE, FAKE, FAKE, 64, 32, FAKE,
-             tb.TK_BF16, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG            # max_seq_len < seq
+             tb.TK_BF16, 0.1, 1, None, 0, None) == tb.TK_ERR_INVALID_ARG      # max_seq_len < seq
     assert P(ctypes.byref(d), None, FAKE, FAKE, None, None, FAKE, FAKE, FAKE, 64, 256, FAKE,
-             tb.TK_BF16, 0.1, 1, None) == tb.TK_ERR_INVALID_ARG            # q is NULL
+             tb.TK_BF16, 0.1, 1, None, 0, None) == tb.TK_ERR_INVALID_ARG      # q is NULL
     assert P(ctypes.byref(d), FAKE, FAKE, FAKE, None, None, FAKE, FAKE, FAKE, 64, 256, FAKE,
-             tb.TK_BF16, -1.0, 1, None) == tb.TK_ERR_INVALID_ARG           # scale <= 0
+             tb.TK_BF16, -1.0, 1, None, 0, None) == tb.TK_ERR_INVALID_ARG     # scale <= 0
     assert P(ctypes.byref(d), None, None, None, None, None, None, None, None, 0, 0, None,
-             tb.TK_BF16, 0.1, 1, None) == tb.TK_OK                          # empty chunk: no-op
+             tb.TK_BF16, 0.1, 1, None, 0, None) == tb.TK_OK                    # empty chunk: no-op
+    # int8 keys need a workspace: NULL, misaligned or too small is rejected
+    # before anything is launched
+    need = lib.tk_prefill_cached_workspace_size(ctypes.byref(d8), 256)
+    assert need > 0
+    args = (ctypes.byref(d8), FAKE, FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, 64, 256, FAKE,
+            tb.TK_BF16, 0.1, 1)
+    assert P(*args, None, need, None) == tb.TK_ERR_WORKSPACE
+    assert P(*args, ctypes.c_void_p(0x10010), need, None) == tb.TK_ERR_WORKSPACE
+    assert P(*args, FAKE, need - 1, None) == tb.TK_ERR_WORKSPACE
+    assert "needed" in tb.tk_last_error()
+
+
+@pytest.mark.parametrize("r,k_dtype,two_planes", [
+    (32, tb.TK_I8, True), (32, tb.TK_I4, True), (64, tb.TK_I8, True), (128, tb.TK_I8, False),
+    (128, tb.TK_I4, False), (16, tb.TK_I8, True)])
+def test_prefill_cached_workspace_size(lib, r, k_dtype, two_planes):
+    """Widened keys: hi and lo bf16 planes of r per token and kv head (r <= 64), or one
+    bf16 plane and an fp32 scale (r = 128), over min(max_seq_len, cache tokens) rows
+    rounded up to 4; nothing for bf16 keys, int4 keys with r < 32 or a bad descriptor."""
+    size = lib.tk_prefill_cached_workspace_size
+    d = _desc(r=r, k_dtype=k_dtype)                 # batch 2, h_kv 2, capacity 256
+    for max_len, rows in ((100, 100), (101, 104), (1000, 256)):
+        per_row = 4 * r if two_planes else 2 * r + 4
+        assert size(ctypes.byref(d), max_len) == 2 * 2 * rows * per_row
+    assert size(ctypes.byref(_desc(r=r)), 100) == 0                       # bf16 keys
+    assert size(ctypes.byref(_desc(r=16, k_dtype=tb.TK_I4)), 100) == 0    # int4 needs r >= 32
+    assert size(ctypes.byref(_desc(r=24, k_dtype=tb.TK_I8)), 100) == 0    # invalid descriptor
+    assert size(ctypes.byref(d), 0) == 0
+    paged = _desc(r=r, k_dtype=k_dtype, capacity=0, page_size=16, num_pages=64, max_pages_per_seq=8)
+    per_row = 4 * r if two_planes else 2 * r + 4
+    assert size(ctypes.byref(paged), 1000) == 2 * 2 * 128 * per_row      # 8 pages of 16 tokens
 
 
 def test_forward_and_backward_validation(lib):
