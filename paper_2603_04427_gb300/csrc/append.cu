@@ -9,11 +9,12 @@
 // One warp per run of kRows consecutive tokens of one (b, g): every 16-byte
 // piece of the run's bf16 rows is loaded before any is stored, so a warp has
 // kRows rows in flight (one row per warp leaves the copy far below the HBM
-// rate: too few bytes in flight per SM).  Quantised keys are then written row
-// by row (a warp max-reduction gives each row's amax).
+// rate: too few bytes in flight per SM).  Quantised keys take the same
+// 16-byte pieces: each lane quantises its 8 elements, and the lanes that hold
+// one row (r/8 neighbours) combine their amax by shuffles; the arithmetic per
+// element is that of kv_row.cuh's quantiser, so the codes are identical.
 #include "common.cuh"
 #include "kernels.h"
-#include "kv_row.cuh"
 
 namespace tk {
 namespace {
@@ -75,13 +76,11 @@ __global__ void __launch_bounds__(kWarps * 32) append_kernel(const AppendParams 
     vdst[i] = c < kRows * NV ? dst_row(c / NV) : -1;
     if (vdst[i] >= 0) vr[i] = vs[c];
   }
-  if constexpr (KF == 0) {
 #pragma unroll
-    for (int i = 0; i < PK; ++i) {
-      const int c = lane + 32 * i;
-      kdst[i] = c < kRows * NK ? dst_row(c / NK) : -1;
-      if (kdst[i] >= 0) kr[i] = ks[c];
-    }
+  for (int i = 0; i < PK; ++i) {
+    const int c = lane + 32 * i;
+    kdst[i] = c < kRows * NK ? dst_row(c / NK) : -1;
+    if (kdst[i] >= 0) kr[i] = ks[c];
   }
 #pragma unroll
   for (int i = 0; i < PV; ++i)
@@ -91,12 +90,44 @@ __global__ void __launch_bounds__(kWarps * 32) append_kernel(const AppendParams 
     for (int i = 0; i < PK; ++i)
       if (kdst[i] >= 0) kd[kdst[i] * NK + (lane + 32 * i) % NK] = kr[i];
   } else {
-#pragma unroll 1
-    for (int i = 0; i < kRows; ++i) {
-      const long long d = dst_row(i);
-      if (d >= 0)
-        write_k_row<R, KF>(p.k, p.k_scale, static_cast<size_t>(d),
-                           static_cast<const unsigned char*>(p.k_new) + (src0 + i) * 2 * R, lane);
+    // symmetric per-token quantisation (Section 6): scale = amax / Q (IEEE
+    // division), code = clamp(rint(x / scale), -Q, Q), 0 when amax is 0
+    constexpr float Q = KF == 1 ? 127.0f : 7.0f;
+#pragma unroll
+    for (int i = 0; i < PK; ++i) {
+      const uint32_t w[4] = {kr[i].x, kr[i].y, kr[i].z, kr[i].w};
+      float x[8];
+      float amax = 0.f;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        x[e] = __uint_as_float(e % 2 == 0 ? w[e / 2] << 16 : w[e / 2] & 0xffff0000u);  // bf16 -> f32
+        amax = fmaxf(amax, fabsf(x[e]));
+      }
+      // the NK lanes of one row are neighbours (c = lane + 32 i, NK divides 32)
+#pragma unroll
+      for (int off = NK / 2; off >= 1; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+      if (kdst[i] < 0) continue;
+      const float scale = amax / Q;
+      int code[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        float cf = 0.f;
+        if (scale != 0.f) cf = fminf(fmaxf(rintf(x[e] / scale), -Q), Q);
+        code[e] = static_cast<int>(cf);
+      }
+      const int piece = (lane + 32 * i) % NK;
+      if constexpr (KF == 1) {
+        uint2 o;
+        o.x = (code[0] & 0xFF) | (code[1] & 0xFF) << 8 | (code[2] & 0xFF) << 16 | (code[3] & 0xFF) << 24;
+        o.y = (code[4] & 0xFF) | (code[5] & 0xFF) << 8 | (code[6] & 0xFF) << 16 | (code[7] & 0xFF) << 24;
+        *reinterpret_cast<uint2*>(static_cast<int8_t*>(p.k) + kdst[i] * R + piece * 8) = o;
+      } else {
+        uint32_t o = 0;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) o |= static_cast<uint32_t>(code[e] & 0xF) << (4 * e);
+        *reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(p.k) + kdst[i] * (R / 2) + piece * 4) = o;
+      }
+      if (piece == 0) p.k_scale[kdst[i]] = scale;
     }
   }
 }
