@@ -885,15 +885,17 @@ def main():
         # training backward and chunked prefill of the 7B shape
         pw = wl.MHA7B_PREFILL
         bw = measure_backward(pw, 10, device, torch)
-        extra[pw.name.replace("prefill", "backward")] = dict(
-            pw.as_config(), kernel="bwd_tc_kernel<32,128> (tcgen05)", ms=r3(bw["ms"]),
+        bname = pw.name.replace("prefill", "backward")
+        extra[bname] = dict(
+            pw.as_config(), workload=bname, kernel="bwd_tc_kernel<32,128> (tcgen05)", ms=r3(bw["ms"]),
             tflops=r3(bw["tflops"]), frac=r3(bw["tflops"] / peaks["bf16_tflops"]),
             flops_per_call=bw["flops_per_call"], launches=bw["launches"])
         cw = wl.CHUNKED_PREFILL
         for kf in ("bf16", "int8"):
             cp = measure_chunked_prefill(cw, 20, device, torch, k_fmt=kf)
             name = cw.name if kf == "bf16" else cw.name + "_int8_keys"
-            extra[name] = dict(cw.as_config(), k_dtype=kf, ms=r3(cp["ms"]), tflops=r3(cp["tflops"]),
+            extra[name] = dict(cw.as_config(), workload=name, k_dtype=kf, ms=r3(cp["ms"]),
+                               tflops=r3(cp["tflops"]),
                                frac=r3(cp["tflops"] / peaks["bf16_tflops"]),
                                append_ms=r3(cp["append_ms"]), flops_per_call=cp["flops_per_call"],
                                launches=cp["launches"])
