@@ -157,9 +157,8 @@ def test_7b_chunk_after_4096_cached_sampled():
     parity_bf16(np.stack(got), np.stack(ref), what="7b cached chunk sampled")
 
 
-@pytest.mark.parametrize("kfmt,r,dv", [("int8", 16, 64), ("int8", 32, 128), ("int8", 64, 64),
-                                       ("int8", 128, 128), ("int4", 32, 128), ("int4", 64, 128),
-                                       ("int4", 128, 64)])
+@pytest.mark.parametrize("kfmt,r,dv", [(k, r, dv) for k in ("int8", "int4") for r in (16, 32, 64, 128)
+                                       for dv in (64, 128) if not (k == "int4" and r < 32)])
 def test_quantised_cached_prefill_matches_oracle(kfmt, r, dv):
     require_gpu()
     B, hq, hkv, S = 3, 8, 2, 300
@@ -181,9 +180,10 @@ def test_quantised_cached_prefill_matches_oracle(kfmt, r, dv):
 
 @pytest.mark.parametrize("kfmt", ["int8", "int4"])
 @pytest.mark.parametrize("ps", [16, 64, 256])
-def test_quantised_cached_prefill_paged_equals_contiguous_bitwise(kfmt, ps):
+@pytest.mark.parametrize("r,dv", [(32, 128), (128, 64)])
+def test_quantised_cached_prefill_paged_equals_contiguous_bitwise(kfmt, ps, r, dv):
     require_gpu()
-    B, hq, hkv, r, dv, S = 3, 8, 2, 32, 128, 257
+    B, hq, hkv, S = 3, 8, 2, 257
     L0 = [5, 130, 640]
     a = _setup(B, hq, hkv, r, dv, L0, S, seed=23, kfmt=kfmt)
     p = _setup(B, hq, hkv, r, dv, L0, S, seed=23, ps=ps, kfmt=kfmt)
@@ -193,6 +193,70 @@ def test_quantised_cached_prefill_paged_equals_contiguous_bitwise(kfmt, ps):
     ref = oa.attention_prefill_cached(f64(a[1]), _keys_for_oracle(a[4], kfmt), f64(a[5]), L0,
                                       1 / math.sqrt(r))
     parity(f64(out_p), ref, what=f"paged {kfmt} ps={ps}")
+
+
+def _bf16_rne(x):
+    """float32 array -> bf16 bit patterns (uint16), rounded to nearest even (finite x)."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    return ((u + 0x7FFF + ((u >> 16) & 1)) >> 16).astype(np.uint16)
+
+
+@pytest.mark.parametrize("kfmt,r,dv", [("int8", 32, 128), ("int4", 64, 128), ("int8", 16, 64),
+                                       ("int8", 128, 64), ("int4", 128, 128)])
+def test_widened_keys_in_the_workspace(kfmt, r, dv):
+    """The workspace after a call holds every context token's key widened as
+    tk_prefill_cached_workspace_size documents: for r <= 64, plane 0 = hi =
+    bf16(scale * code) and plane 1 = lo = bf16(scale * code - hi) (the product in
+    fp32, both roundings to nearest even), so hi + lo is within 2^-17 of the
+    product; for r = 128, the codes as exact bf16 and the fp32 scales.  Computed
+    here independently from the cache's codes and scales."""
+    require_gpu()
+    B, hq, hkv, S = 2, 4, 2, 200
+    L0 = [0, 333]
+    cache, q, kn, vn, K, V, n = _setup(B, hq, hkv, r, dv, L0, S, seed=61 + r, kfmt=kfmt)
+    ws = tb.prefill_cached_workspace(cache, n)
+    out = torch.empty(B, hq, S, dv, dtype=torch.float32, device="cuda")
+    sl = torch.tensor(L0, dtype=torch.int32, device="cuda")
+    tb.tk_attn_prefill_cached(cache, q, kn, vn, sl, n, out, workspace=ws)
+    torch.cuda.synchronize()
+    assert tb.tk_get_device_error() == 0
+    rows = (n + 3) // 4 * 4
+    plane = B * hkv * rows * r
+    w = ws.cpu().numpy()
+    p0 = w[:2 * plane].view(np.uint16).reshape(B, hkv, rows, r)
+    codes = cache.k.cpu().numpy()
+    codes = codes if kfmt == "int8" else oc.unpack_int4(codes)
+    scales = cache.k_scale.cpu().numpy()
+    two = r <= 64
+    assert ws.numel() == (4 * plane if two else 2 * plane + 4 * B * hkv * rows)
+    for b, l0 in enumerate(L0):
+        c = codes[b, :, :l0 + S].astype(np.float32)
+        s = scales[b, :, :l0 + S]
+        if two:
+            x = c * s[..., None]                                   # fp32 product
+            hi = _bf16_rne(x)
+            lo = _bf16_rne(x - (hi.astype(np.uint32) << 16).view(np.float32))
+            p1 = w[2 * plane:4 * plane].view(np.uint16).reshape(B, hkv, rows, r)
+            assert np.array_equal(p0[b, :, :l0 + S], hi)
+            assert np.array_equal(p1[b, :, :l0 + S], lo)
+            back = (hi.astype(np.uint32) << 16).view(np.float32).astype(np.float64) + \
+                (lo.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+            exact = c.astype(np.float64) * s[..., None].astype(np.float64)
+            assert np.all(np.abs(back - exact) <= 2.0 ** -17 * np.abs(exact) + 2.0 ** -24 * np.abs(exact))
+        else:
+            assert np.array_equal(p0[b, :, :l0 + S], _bf16_rne(c))  # small integers: exact
+            sp = w[2 * plane:2 * plane + 4 * B * hkv * rows].view(np.float32).reshape(B, hkv, rows)
+            assert np.array_equal(sp[b, :, :l0 + S].view(np.uint32), s.view(np.uint32))
+
+
+def test_quantised_prefill_rejects_a_short_workspace():
+    require_gpu()
+    cache, q, kn, vn, K, V, n = _setup(1, 4, 2, 32, 128, [64], 128, seed=5, kfmt="int8")
+    ws = tb.prefill_cached_workspace(cache, n)
+    out = torch.empty(1, 4, 128, 128, dtype=torch.float32, device="cuda")
+    sl = torch.tensor([64], dtype=torch.int32, device="cuda")
+    with pytest.raises(RuntimeError, match="TK_ERR_WORKSPACE"):
+        tb.tk_attn_prefill_cached(cache, q, kn, vn, sl, n, out, workspace=ws[:-256])
 
 
 @pytest.mark.parametrize("kfmt,ps", [("bf16", 0), ("int8", 0), ("bf16", 64), ("int4", 16)])
