@@ -543,10 +543,13 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       // natural-log logsumexp of the row's scaled scores (for the backward):
       // sum_j exp(scale s_j) = 2^m_used * l
       if (p.lse && store) p.lse[static_cast<size_t>(bh) * p.S + row] = (m_used + log2f(l)) * 0.69314718055994531f;
+      // the whole O row with one TMEM wait (the score registers are free by now)
+      uint32_t o[DV];
+      if constexpr (DV == 128) tmem_ld128(tO + lane_off, o);
+      else tmem_ld64(tO + lane_off, o);
 #pragma unroll
       for (int c = 0; c < DV / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld32(tO + lane_off + 32 * c, v);
+        const uint32_t* v = o + 32 * c;
         if (store) {
           if (p.out_f32) {
             float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.out) + obase + 32 * c);
