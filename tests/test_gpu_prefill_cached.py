@@ -195,6 +195,24 @@ def test_quantised_cached_prefill_paged_equals_contiguous_bitwise(kfmt, ps, r, d
     parity(f64(out_p), ref, what=f"paged {kfmt} ps={ps}")
 
 
+@pytest.mark.parametrize("kfmt,r,dv,L0,S,causal,bf16_out", [
+    ("int8", 32, 128, [128, 0], 128, True, True),     # contexts end on a tile boundary
+    ("int4", 64, 128, [256, 3], 129, False, False),   # full attention over the context
+    ("int8", 128, 64, [0, 1], 1, True, False),        # a one-token chunk (scales in the softmax)
+    ("int4", 32, 64, [1000, 17], 64, False, True),
+])
+def test_quantised_cached_prefill_edge_cases(kfmt, r, dv, L0, S, causal, bf16_out):
+    require_gpu()
+    B, hq, hkv = len(L0), 4, 2
+    cache, q, kn, vn, K, V, n = _setup(B, hq, hkv, r, dv, L0, S, seed=71 + S, kfmt=kfmt)
+    out = _run(cache, q, kn, vn, L0, n, dtype=torch.bfloat16 if bf16_out else torch.float32,
+               causal=causal)
+    ref = oa.attention_prefill_cached(f64(q), _keys_for_oracle(K, kfmt), f64(V), L0,
+                                      1 / math.sqrt(r), causal=causal)
+    check = parity_bf16 if bf16_out else parity
+    check(f64(out), ref, what=f"{kfmt} r={r} L0={L0} S={S} causal={causal}")
+
+
 def _bf16_rne(x):
     """float32 array -> bf16 bit patterns (uint16), rounded to nearest even (finite x)."""
     u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
