@@ -717,8 +717,8 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--headline-only", action="store_true",
                     help="skip the secondary workloads and the CPU baseline")
-    ap.add_argument("--only", choices=("decode", "prefill", "chunked", "backward", "gpt2", "paged",
-                                       "int8", "cpu"),
+    ap.add_argument("--only", choices=("decode", "prefill", "chunked", "chunked-r", "backward", "gpt2",
+                                       "paged", "int8", "cpu"),
                     help="run one secondary workload alone (for profiling) and print its result; "
                          "cpu: the oracle's time on every workload")
     args = ap.parse_args()
@@ -759,6 +759,17 @@ def main():
         elif args.only == "chunked":
             for kf in ("bf16", "int8", "int4"):
                 res[kf] = measure_chunked_prefill(wl.CHUNKED_PREFILL, args.steps, device, torch, k_fmt=kf)
+        elif args.only == "chunked-r":
+            # the same chunk at every thin-key width, bf16 and int8 keys
+            import dataclasses
+            rows = []
+            for r in (16, 32, 64, 128):
+                cw = dataclasses.replace(wl.CHUNKED_PREFILL, r=r)
+                for kf in ("bf16", "int8"):
+                    cp = measure_chunked_prefill(cw, args.steps, device, torch, k_fmt=kf)
+                    rows.append([r, kf, round(cp["ms"], 4), round(cp["tflops"], 1),
+                                 round(cp["tflops"] / peaks["bf16_tflops"], 4)])
+            res["sweep"] = {"cols": ["r", "k_dtype", "ms", "TFLOP/s", "frac"], "rows": rows}
         elif args.only == "gpt2":
             res.update(measure_gpt2_layer(wl.GPT2_LAYER, args.steps, device, torch))
         elif args.only == "decode":

@@ -103,15 +103,16 @@ struct PCfg {
   static constexpr int OFF_Q = 0;                        // two Q tiles
   static constexpr int OFF_K = 2 * QBA;
   static constexpr int KBA = (KB + 1023) / 1024 * 1024;
-  // K tiles per stage: 2 for quantised keys widened to hi + lo (where two
-  // stages of them fit), else 1 (bf16 keys, or exact bf16 codes whose scales
-  // the softmax applies)
-  static constexpr int KT = (KF != 0 && 2 * QBA + 2 * (2 * KBA + VB) + 2048 <= 200 * 1024) ? 2 : 1;
+  // K tiles per stage: 2 for quantised keys widened to hi + lo where a
+  // 3-stage ring of them fits the 227 KB a CTA may hold (a 2-stage ring was
+  // measured 40 % slower at r = 64), else 1 (bf16 keys, or exact bf16 codes
+  // whose scales the softmax applies)
+  static constexpr int KT = (KF != 0 && 2 * QBA + 3 * (2 * KBA + VB) + 2048 <= 227 * 1024) ? 2 : 1;
   static constexpr bool SCALE_IN_SOFTMAX = KF != 0 && KT == 1;
   static constexpr int SCB = SCALE_IN_SOFTMAX ? kBN * 4 : 0;  // a tile's key scales
   static constexpr int VOFF = KT * KBA;              // V tile offset in a stage
   static constexpr int STAGE = VOFF + VB;
-  static constexpr int NST = (2 * QBA + 3 * (STAGE + SCB) + 2048 <= 200 * 1024) ? 3 : 2;
+  static constexpr int NST = (KT == 2 || 2 * QBA + 3 * (STAGE + SCB) + 2048 <= 200 * 1024) ? 3 : 2;
   static constexpr int OFF_SC = OFF_K + NST * STAGE;
   static constexpr int OFF_BAR = OFF_SC + NST * SCB;
   static constexpr int SMEM = OFF_BAR + 256 + 1024;      // + slack to align the base to 1 KB
