@@ -501,11 +501,11 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
       const float2 sl2x2 = make_float2(sl2, sl2), negm2 = make_float2(-m_used, -m_used);
       float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                        make_float2(0.f, 0.f)};
+      static_assert(kParts == 2, "two key ranges of P");
+      // pairs [i0, i1) of key range c into pk[i0 .. i1)
+      auto compute = [&](int c, int i0, int i1, uint32_t* pk) {
 #pragma unroll
-      for (int c = 0; c < kParts; ++c) {
-        uint32_t pk[kPartPairs];
-#pragma unroll
-        for (int i = 0; i < kPartPairs; ++i) {
+        for (int i = i0; i < i1; ++i) {
           const int e = 2 * kPartPairs * c + 2 * i;
           const float2 t = ffma2(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])),
                                  sl2x2, negm2);
@@ -514,23 +514,34 @@ prefill_kernel(const __grid_constant__ Maps maps, const PrefillParams p) {
           __nv_bfloat162 b2 = __floats2bfloat162_rn(pr.x, pr.y);  // low half = column e
           pk[i] = *reinterpret_cast<uint32_t*>(&b2);
         }
-        tmem_st<kPartPairs>(tS + lane_off + kPartPairs * c, pk);
-        if (c == 0 && j > 0 && __any_sync(0xffffffffu, resc)) {
-          // O *= alpha before any P V product of this tile accumulates into it; the
-          // previous one is complete (the S_j commit covers it)
-#pragma unroll 1
-          for (int cc = 0; cc < DV / 16; ++cc) {
-            uint32_t o[16];
-            tmem_ld16(tO + lane_off + 16 * cc, o);
-#pragma unroll
-            for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-            tmem_st16(tO + lane_off + 16 * cc, o);
-          }
-        }
+      };
+      auto publish = [&](int c) {
         tmem_wait_st();
         tc_fence_before();
         mbar_arrive(&p_full[kParts * x + c]);
+      };
+      uint32_t pk0[kPartPairs], pk1[kPartPairs];
+      compute(0, 0, kPartPairs, pk0);
+      tmem_st<kPartPairs>(tS + lane_off, pk0);
+      if (j > 0 && __any_sync(0xffffffffu, resc)) {
+        // O *= alpha before any P V product of this tile accumulates into it; the
+        // previous one is complete (the S_j commit covers it)
+#pragma unroll 1
+        for (int cc = 0; cc < DV / 16; ++cc) {
+          uint32_t o[16];
+          tmem_ld16(tO + lane_off + 16 * cc, o);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+          tmem_st16(tO + lane_off + 16 * cc, o);
+        }
       }
+      // the first half of range 1 while range 0's store lands, then range 0 is
+      // published; same arithmetic and order of sums as range by range
+      compute(1, 0, kPartPairs / 2, pk1);
+      publish(0);
+      compute(1, kPartPairs / 2, kPartPairs, pk1);
+      tmem_st<kPartPairs>(tS + lane_off + kPartPairs, pk1);
+      publish(1);
       const float2 s01 = fadd2(acc[0], acc[1]), s23 = fadd2(acc[2], acc[3]);
       l += (s01.x + s01.y) + (s23.x + s23.y);
     }
