@@ -267,6 +267,32 @@ def test_widened_keys_in_the_workspace(kfmt, r, dv):
             assert np.array_equal(sp[b, :, :l0 + S].view(np.uint32), s.view(np.uint32))
 
 
+def test_workspace_reused_across_calls_and_shapes():
+    """One workspace, large enough for the biggest call, serves calls of other
+    shapes and key formats in stream order: every result equals, bit for bit,
+    the same call with a fresh workspace of its own."""
+    require_gpu()
+    cases = [("int8", 64, 128, [500, 20], 300), ("int4", 32, 64, [0, 77], 130),
+             ("int8", 128, 64, [128, 1], 64), ("int8", 64, 128, [500, 20], 300)]
+    sizes = []
+    for kfmt, r, dv, L0, S in cases:
+        cache, *_rest, n = _setup(len(L0), 4, 2, r, dv, L0, S, seed=3, kfmt=kfmt)
+        sizes.append(tb.prefill_cached_workspace(cache, n).numel())
+    shared = torch.full((max(sizes),), 0x7F, dtype=torch.uint8, device="cuda")  # garbage
+    for i, (kfmt, r, dv, L0, S) in enumerate(cases):
+        a = _setup(len(L0), 4, 2, r, dv, L0, S, seed=90 + i, kfmt=kfmt)
+        b = _setup(len(L0), 4, 2, r, dv, L0, S, seed=90 + i, kfmt=kfmt)
+        sl = torch.tensor(L0, dtype=torch.int32, device="cuda")
+        outs = []
+        for (cache, q, kn, vn, K, V, n), ws in ((a, shared), (b, None)):
+            out = torch.empty(len(L0), 4, S, dv, dtype=torch.float32, device="cuda")
+            tb.tk_attn_prefill_cached(cache, q, kn, vn, sl, n, out, workspace=ws)
+            outs.append(out)
+        torch.cuda.synchronize()
+        assert tb.tk_get_device_error() == 0
+        assert torch.equal(outs[0], outs[1]), (kfmt, r, dv)
+
+
 def test_quantised_prefill_rejects_a_short_workspace():
     require_gpu()
     cache, q, kn, vn, K, V, n = _setup(1, 4, 2, 32, 128, [64], 128, seed=5, kfmt="int8")
